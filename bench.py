@@ -1,0 +1,358 @@
+"""Benchmark of one mixed prefill/decode paged-attention step on GB300.
+
+A step is the whole hot path over one synthetic batch: KV append of the
+step's new tokens, then attention of every query (prefill chunk + decodes)
+through the C ABI. Default workload: the Qwen2.5-7B-shaped co-located step
+(one 2048-token prefill chunk on a cached prefix ~ U[0, 8192] plus 128
+decodes with log-normal contexts, 28/4 heads, d 128, block size 16).
+
+Prints one JSON line (rank 0): query tokens/s for the whole job, the roofline
+fraction of the dominant kernel, the end-to-end figure through host buffers,
+the oracle's CPU time on the host cores, and clocks seen during the timed
+region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 oracle on the host cores
+
+Under torchrun each rank runs an independent replica (seed + rank): the path
+has no exchange step, so there is no collective on the data path.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "mixed PD attention query tokens/s at 1 GB300; % of max(FLOP,HBM) roofline"
+UNIT = "query tokens/s"
+L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle reasons sampled every 200 ms while active."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def _sample_rows(batch, target_pairs: int):
+    """Evenly spaced query rows whose visible pairs sum to about target_pairs."""
+    T = batch.num_tokens
+    seq_of = np.repeat(np.arange(batch.num_seqs), batch.query_len)
+    idx = np.arange(T) - batch.query_start[seq_of]
+    pos = batch.context_len[seq_of] - batch.query_len[seq_of] + idx
+    row_pairs = (pos + 1).astype(np.int64)
+    total = int(row_pairs.sum())
+    frac = min(1.0, max(target_pairs, 1) / total)
+    n = max(1, int(round(T * frac)))
+    rows = np.unique(np.linspace(0, T - 1, n).round().astype(np.int64))
+    return rows, int(row_pairs[rows].sum()), total
+
+
+def cpu_baseline(batch, target_seconds: float = 15.0, reps: int = 1):
+    """Time the fp64 oracle on a bounded, evenly spaced sample of the step's
+    query rows on all host cores; extrapolate to the whole step by visible
+    (query, key) pairs."""
+    import oracle
+    threads = oracle.max_threads()
+    sh = batch.shape
+    t0 = time.perf_counter()
+    kc = oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping)
+    vc = None if sh.latent else oracle.kv_append(batch.v_cache, batch.v_new, batch.slot_mapping)
+    t_append = time.perf_counter() - t0
+    kw = dict(num_q_heads=sh.num_q_heads, num_kv_heads=sh.num_kv_heads, head_dim_qk=sh.head_dim_qk,
+              head_dim_v=sh.head_dim_v, block_size=sh.block_size, latent=sh.latent)
+    # calibrate the oracle's pair rate: grow a sample until it takes >= 0.2 s
+    target = max(1, W.pairs(batch) // 4096)
+    while True:
+        rows, sp, total = _sample_rows(batch, target_pairs=target)
+        t0 = time.perf_counter()
+        oracle.attention(batch.query_len, batch.context_len, batch.block_table, batch.q, kc, vc,
+                         tokens=rows, **kw)
+        dt = time.perf_counter() - t0
+        if dt >= 0.2 or sp >= total:
+            break
+        target *= 4
+    rate = sp / max(dt, 1e-6)
+    rows, sp, total = _sample_rows(batch, target_pairs=int(rate * target_seconds))
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        oracle.attention(batch.query_len, batch.context_len, batch.block_table, batch.q, kc, vc,
+                         tokens=rows, **kw)
+        times.append(time.perf_counter() - t0)
+    t_sample = statistics.median(times)
+    t_step = t_append + t_sample * total / sp
+    return {"value": batch.num_tokens / t_step, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": (f"{len(rows)} of {batch.num_tokens} query rows (every ~{batch.num_tokens // max(len(rows), 1)}th, "
+                       f"{sp / total:.4f} of the visible pairs), fp64 C oracle with OpenMP; "
+                       f"step time extrapolated by pairs plus the full KV append"),
+            "sample_seconds": t_sample, "step_seconds_extrapolated": t_step}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return 0
+    batch = W.make_batch(args.workload, seed=args.seed)
+    per = []
+    for i in range(args.warmup + args.steps):
+        r = cpu_baseline(batch, target_seconds=args.ref_seconds)
+        if i >= args.warmup:
+            per.append(r)
+    step_s = statistics.median(x["step_seconds_extrapolated"] for x in per)
+    value = batch.num_tokens / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": args.workload, "seed": args.seed},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": per[0]["cores"], "kind": "oracle",
+                             "sample": per[0]["sample"]},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_fnpu(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    fnpu.load()
+    peaks = _peaks()
+
+    batch = W.make_batch(args.workload, seed=args.seed + rank)
+    work = W.algorithmic_work(batch)
+    opts = fnpu.PlanOpts(args.split, args.decode_share, 0, args.flags)
+    st = DeviceStep(batch, opts=opts, device=str(dev))
+    info = st.plan.info()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    for _ in range(args.warmup):
+        st.run()
+    torch.cuda.synchronize(dev)
+    if fnpu.plan_check(st.plan) != fnpu.FNPU_OK or fnpu.check() != fnpu.FNPU_OK:
+        raise RuntimeError("device error flag raised during warm-up")
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clocks:
+        for i in range(K):
+            flush.zero_()  # evict L2 between timed steps (outside the events)
+            ev[i][0].record(stream)
+            st.append()
+            ev[i][1].record(stream)
+            st.attend()
+            ev[i][2].record(stream)
+        torch.cuda.synchronize(dev)
+        if ws > 1:
+            dist.barrier()
+    clk = clocks.summary()
+    t_append = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
+    t_attn = [ev[i][1].elapsed_time(ev[i][2]) for i in range(K)]
+    step_ms = sum(a + b for a, b in zip(t_append, t_attn)) / K
+    attn_ms = sum(t_attn) / K
+    if ws > 1:
+        t = torch.tensor([step_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        step_ms = float(t.item())
+
+    # end to end through host buffers: H2D of the step's inputs, append + attention,
+    # D2H of the outputs, all inside the timed region
+    bf = torch.bfloat16
+    h_q = torch.from_numpy(batch.q).view(bf).pin_memory()
+    h_k = torch.from_numpy(batch.k_new).view(bf).pin_memory()
+    h_v = None if batch.v_new is None else torch.from_numpy(batch.v_new).view(bf).pin_memory()
+    h_s = torch.from_numpy(batch.slot_mapping).pin_memory()
+    h_o = torch.empty(st.out.shape, dtype=bf).pin_memory()
+    h_l = torch.empty(st.lse.shape, dtype=torch.float32).pin_memory()
+    h2d = sum(x.numel() * x.element_size() for x in (h_q, h_k, h_v, h_s) if x is not None)
+    d2h = h_o.numel() * h_o.element_size() + h_l.numel() * h_l.element_size()
+    e2e_ms = []
+    for i in range(args.warmup + K):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        st.q.copy_(h_q, non_blocking=True)
+        st.k_new.copy_(h_k, non_blocking=True)
+        if h_v is not None:
+            st.v_new.copy_(h_v, non_blocking=True)
+        st.slot_mapping.copy_(h_s, non_blocking=True)
+        st.run()
+        h_o.copy_(st.out, non_blocking=True)
+        h_l.copy_(st.lse, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        if i >= args.warmup:
+            e2e_ms.append(a.elapsed_time(b))
+    e2e = sum(e2e_ms) / len(e2e_ms)
+    if ws > 1:
+        t = torch.tensor([e2e], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e = float(t.item())
+
+    # roofline of the dominant kernel work (the attention launch): algorithmic
+    # FLOPs and bytes per run / measured duration
+    F = work["flops"]
+    B_attn = work["bytes"] - work["append_bytes"] - 8 * batch.num_tokens
+    t_s = attn_ms * 1e-3
+    tf_time = F / (peaks["bf16_tflops"] * 1e12)
+    hb_time = B_attn / (peaks["hbm_gbs"] * 1e9)
+    if tf_time >= hb_time:
+        roof = {"bound": "tensor", "achieved": F / t_s / 1e12, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": B_attn / t_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = args.traffic
+    roof["peak_source"] = peaks["source"] + " burst"
+    step_roof = max(F / (peaks["bf16_tflops"] * 1e12), work["bytes"] / (peaks["hbm_gbs"] * 1e9))
+    step_roof_sus = max(F / (peaks["bf16_tflops_sustained"] * 1e12), work["bytes"] / (peaks["hbm_gbs"] * 1e9))
+
+    T = batch.num_tokens
+    line = {
+        "metric": METRIC, "value": ws * T / (step_ms * 1e-3), "unit": UNIT, "n_gpus": ws,
+        "steps": K, "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T,
+                   "num_seqs": batch.num_seqs, "prefill_ctx": int(batch.context_len[0]),
+                   "flops": F, "bytes": work["bytes"], "l2": "flushed between timed steps (512 MB write)",
+                   "plan": info},
+        "roofline": roof,
+        "roofline_step_frac": {"burst": step_roof / (step_ms * 1e-3),
+                               "sustained": step_roof_sus / (step_ms * 1e-3),
+                               "denominator": "max(F/bf16 peak, B/HBM peak) of measured"},
+        "kernel_ms": {"append": sum(t_append) / K, "attention": attn_ms},
+        "e2e": {"value": ws * T / (e2e * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
+        "gpu_launches": K * (1 + info["launches_per_run"]),
+        "clocks": clk,
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(batch, target_seconds=args.ref_seconds)
+    elif rank == 0:
+        line["cpu_baseline"] = None
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="fnpu", choices=["fnpu", "reference"])
+    ap.add_argument("--workload", default="qwen_coloc", choices=list(W.CONFIG_NAMES))
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--split", type=int, default=0, help="decode split keys (0 = planner)")
+    ap.add_argument("--decode-share", type=int, default=0)
+    ap.add_argument("--flags", type=int, default=0)
+    ap.add_argument("--ref-seconds", type=float, default=15.0)
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="ncu dram bytes per attention launch, if measured for this kernel")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(args.warmup, 3)  # at least three untimed warm-up steps
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_fnpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,172 @@
+/*
+ * fnpu.h -- C ABI of the GB300 mixed prefill/decode paged-attention step.
+ *
+ * One serving step in which prefill chunks and decode queries share the
+ * device and one paged KV pool (the dynamic PD co-location of Sec. 3.4):
+ * prefill is compute-heavy and decode is bound by KV-cache reads (Sec. 1,
+ * Sec. 3.3, Fig. 1-2), so the step interleaves both kinds of work on the same
+ * SMs. A step is
+ *
+ *   fnpu_kv_append          store the step's new K/V rows in their paged slots
+ *   fnpu_mixed_attn_plan    (host) classify sequences by phase and build the
+ *                           work list -- the phase-aware dispatch of Sec. 3.4
+ *   fnpu_mixed_attn_run     causal attention of every query over its sequence's
+ *                           cached keys, one launch on the caller's stream
+ *
+ * As in the paper's control path (Sec. 3.2), calls pass metadata and pointers
+ * only: tensors stay in device memory owned by the caller; the library never
+ * copies them. All entry points are asynchronous on the given CUDA stream
+ * (cudaStream_t passed as void*; NULL = legacy default stream) and return an
+ * fnpu_status; none aborts or prints.
+ *
+ * Math (the paper gives none; this is textbook attention): for sequence s with
+ * query_len q and context_len ctx (ctx counts this step's q new tokens), query
+ * i in [0, q) sits at absolute position pos = ctx - q + i and attends to keys
+ * j = 0..pos of its sequence. Query head h reads kv head h / (Hq / Hkv).
+ *   S_j = scale * <Q[t,h,:], K_j>;  O[t,h,:] = sum_j softmax(S)_j V_j;
+ *   LSE[t,h] = ln sum_j exp(S_j)          (natural log, fp32)
+ * Key j of sequence s lives in block block_table[s][j / bs] at offset j % bs.
+ * Scores and softmax are fp32; QK^T and PV take bf16 operands and fp32
+ * accumulation; O is rounded to bf16 (nearest-even).
+ *
+ * Layouts (row-major, contiguous, bf16 = 16-bit brain float):
+ *   q        bf16 [T, Hq, d_qk]      queries packed sequence by sequence
+ *   k_cache  bf16 [num_blocks, bs, Hkv, d_qk]
+ *   v_cache  bf16 [num_blocks, bs, Hkv, d_v]
+ *   latent (v_in_k_latent = 1, MLA): k_cache bf16 [num_blocks, bs, d_qk],
+ *            Hkv = 1, V = the first d_v columns of each K row, v_cache NULL
+ *   out      bf16 [T, Hq, d_v];  lse fp32 [T, Hq]
+ * All device pointers must be 16-byte aligned.
+ */
+#ifndef FNPU_H_
+#define FNPU_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FNPU_OK = 0,
+    FNPU_EINVAL = -1,          /* bad argument; nothing was launched */
+    FNPU_EUNSUPPORTED = -2,    /* valid but not implemented (head dims etc.) */
+    FNPU_ECUDA = -3,           /* a CUDA runtime call failed */
+    FNPU_EDEVICE_TIMEOUT = -4, /* a bounded device-side wait gave up */
+    FNPU_ENOMEM = -5,          /* device or host allocation failed */
+    FNPU_EDEVICE_RANGE = -6    /* a kernel met an out-of-range slot and skipped it */
+} fnpu_status;
+
+typedef struct {
+    int32_t num_q_heads;   /* Hq, a multiple of num_kv_heads */
+    int32_t num_kv_heads;  /* Hkv (1 for the latent layout) */
+    int32_t head_dim_qk;   /* supported: 64, 128 (split K/V); 576 (latent) */
+    int32_t head_dim_v;    /* = head_dim_qk for split K/V; 512 for latent */
+    int32_t block_size;    /* tokens per KV block (16 or 64 ...), >= 1 */
+    int32_t num_blocks;    /* blocks in the pool */
+    int32_t v_in_k_latent; /* 1: MLA latent cache, V aliases K[:, :d_v] */
+    float softmax_scale;   /* <= 0 selects 1/sqrt(head_dim_qk) */
+} fnpu_attn_desc;
+
+typedef struct fnpu_plan fnpu_plan; /* opaque, owned by the library */
+
+/* Plan options (all zero = defaults). */
+typedef struct {
+    int32_t decode_split_keys; /* keys per decode split item; 0 = chosen by the planner */
+    int32_t decode_share_pct;  /* share of resident work slots that take decode work
+                                  first in the phase-aware schedule; 0 = planner default */
+    int32_t num_sms;           /* SMs to plan for; 0 = the current device's count */
+    int32_t flags;             /* FNPU_PLAN_* bits */
+} fnpu_plan_opts;
+
+#define FNPU_PLAN_SEPARATE_LAUNCHES 1 /* run prefill and decode as separate launches */
+#define FNPU_PLAN_NO_TCGEN05 2        /* prefill on the mma.sync path (comparison only) */
+
+/*
+ * KV append: for each token t in [0, num_tokens) with slot_mapping[t] >= 0,
+ * copy k_new[t] (Hkv*d_qk values; latent: d_qk values) into slot
+ * slot_mapping[t] of k_cache and v_new[t] (Hkv*d_v values) into the same slot
+ * of v_cache, bit-exactly. Slot s means block s / bs, offset s % bs. Negative
+ * slots are padding and are skipped. Must run before fnpu_mixed_attn_run of
+ * the same step: a step's queries see their own new keys.
+ *   desc          attention shape (host pointer)
+ *   k_new, v_new  device bf16 [num_tokens, Hkv, d]; v_new NULL for latent
+ *   slot_mapping  device int64 [num_tokens]
+ *   k_cache, v_cache  device pools as above; v_cache NULL for latent
+ * Errors: FNPU_EINVAL on NULL pointers or bad shape (nothing launched). A slot
+ * >= num_blocks*bs cannot be seen on the host; the kernel skips it and raises
+ * the device error flag, reported as FNPU_EDEVICE_RANGE by fnpu_check().
+ * Duplicate non-negative slots are a caller error (result unspecified).
+ */
+int fnpu_kv_append(const fnpu_attn_desc *desc, const void *k_new, const void *v_new,
+                   const int64_t *slot_mapping, int32_t num_tokens,
+                   void *k_cache, void *v_cache, void *stream);
+
+/*
+ * Build the work list for one step. Host arrays, all of length num_seqs:
+ *   query_len[s] >= 1, context_len[s] >= query_len[s],
+ *   phase[s] = 0 (prefill chunk) or 1 (decode; requires query_len[s] == 1),
+ *   block_table: int32 [num_seqs, block_table_stride]; only the first
+ *   ceil(context_len[s] / bs) entries of row s are read, each < num_blocks.
+ * The phase decides only which queue a sequence's work enters (prefill tiles
+ * on the tensor-core path, decode split items on the bandwidth path), never
+ * the result. The plan copies everything it needs (the block table included)
+ * to its own device workspace with one asynchronous copy on `stream`; the
+ * host arrays may be freed on return. The plan stays valid for any number of
+ * runs with the same metadata and caches of the same shape.
+ * Errors: FNPU_EINVAL for any violated condition above, FNPU_EUNSUPPORTED for
+ * head dims or groupings without a kernel, FNPU_ENOMEM, FNPU_ECUDA.
+ * *out is set only on success.
+ */
+int fnpu_mixed_attn_plan(const fnpu_attn_desc *desc, int32_t num_seqs,
+                         const int32_t *query_len, const int32_t *context_len,
+                         const uint8_t *phase, const int32_t *block_table,
+                         int32_t block_table_stride, void *stream, fnpu_plan **out);
+
+/* As fnpu_mixed_attn_plan, with options (opts may be NULL). */
+int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs,
+                            const int32_t *query_len, const int32_t *context_len,
+                            const uint8_t *phase, const int32_t *block_table,
+                            int32_t block_table_stride, const fnpu_plan_opts *opts,
+                            void *stream, fnpu_plan **out);
+
+/*
+ * Attention for every query of the planned step. q, k_cache, v_cache, out,
+ * lse are device pointers in the layouts above (v_cache NULL for latent).
+ * Enqueues the work on `stream` and returns without synchronising. Runs of
+ * one plan must not overlap on the GPU (they share the plan's split scratch).
+ * Errors: FNPU_EINVAL (NULL pointers), FNPU_ECUDA (launch failure).
+ */
+int fnpu_mixed_attn_run(const fnpu_plan *plan, const void *q, const void *k_cache,
+                        const void *v_cache, void *out, float *lse, void *stream);
+
+/* Synchronise `stream`, then read and clear the plan's device error flag:
+ * FNPU_OK, FNPU_EDEVICE_TIMEOUT or FNPU_ECUDA. */
+int fnpu_plan_check(const fnpu_plan *plan, void *stream);
+
+/* Synchronise `stream`, then read and clear the library-wide device error
+ * flag of the current device (set by fnpu_kv_append on an out-of-range slot):
+ * FNPU_OK, FNPU_EDEVICE_RANGE or FNPU_ECUDA. */
+int fnpu_check(void *stream);
+
+/* Release the plan and its device workspace. Waits for the plan's stream
+ * work to finish first. NULL is ignored. */
+void fnpu_plan_destroy(fnpu_plan *plan);
+
+/* Plan statistics for reporting (host copies; any out pointer may be NULL):
+ * number of prefill tiles, decode split items, kernel launches per run, and
+ * bytes of device workspace the plan holds. */
+int fnpu_plan_info(const fnpu_plan *plan, int32_t *prefill_items, int32_t *decode_items,
+                   int32_t *launches_per_run, int64_t *workspace_bytes);
+
+/* Static description of a status code; never NULL. */
+const char *fnpu_status_str(int status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int fnpu_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FNPU_H_ */

@@ -1,0 +1,382 @@
+// Host side of the C ABI: argument validation, the phase-aware planner and
+// the launch sequence of a run.
+//
+// The planner is the GPU counterpart of the paper's phase-aware dispatch
+// (Sec. 3.4): requests are classified by phase into a prefill queue (tensor
+// work, tiles of query rows) and a decode queue (bandwidth work, split-KV
+// items), and the mix of the two decides how the device is shared. The plan
+// carries metadata only; tensors stay with the caller (Sec. 3.2).
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+#include <mutex>
+#include <set>
+#include <utility>
+#include <vector>
+
+#include "fnpu_internal.h"
+
+struct fnpu_plan {
+    fnpu_attn_desc desc;
+    float scale;
+    int32_t num_seqs = 0;
+    int64_t num_tokens = 0;
+    int32_t bt_width = 0;
+    int32_t num_sms = 0;
+    int32_t flags = 0;
+    int32_t num_ditems = 0, num_pitems = 0, num_groups = 0, num_parts = 0;
+    void *d_ws = nullptr;
+    size_t ws_bytes = 0;
+    void *h_stage = nullptr;
+    fnpu::SeqInfo *d_seqs = nullptr;
+    int32_t *d_bt = nullptr;
+    fnpu::DecodeItem *d_ditems = nullptr;
+    fnpu::PrefillItem *d_pitems = nullptr;
+    int32_t *d_counters = nullptr;
+    int32_t *d_err = nullptr;
+    float *d_part_lse = nullptr;
+    float *d_part_o = nullptr;
+};
+
+namespace fnpu {
+namespace {
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool shape_ok(const fnpu_attn_desc *d, int *status) {
+    *status = FNPU_EINVAL;
+    if (!d) return false;
+    if (d->num_q_heads <= 0 || d->num_kv_heads <= 0 || d->num_q_heads % d->num_kv_heads) return false;
+    if (d->head_dim_qk <= 0 || d->head_dim_v <= 0 || d->block_size <= 0 || d->num_blocks <= 0)
+        return false;
+    if (d->v_in_k_latent) {
+        if (d->num_kv_heads != 1 || d->head_dim_v > d->head_dim_qk) return false;
+    }
+    if ((static_cast<int64_t>(d->head_dim_qk) * 2) % 16 || (static_cast<int64_t>(d->head_dim_v) * 2) % 16)
+        return false;
+    *status = FNPU_OK;
+    return true;
+}
+
+// Kernels exist for split K/V with d in {64, 128} (decode needs G <= 8).
+int kernel_support(const fnpu_attn_desc *d, bool has_decode) {
+    if (d->v_in_k_latent) return FNPU_EUNSUPPORTED;
+    if (d->head_dim_qk != d->head_dim_v) return FNPU_EUNSUPPORTED;
+    if (d->head_dim_qk != 64 && d->head_dim_qk != 128) return FNPU_EUNSUPPORTED;
+    if (has_decode && d->num_q_heads / d->num_kv_heads > 8) return FNPU_EUNSUPPORTED;
+    return FNPU_OK;
+}
+
+}  // namespace
+}  // namespace fnpu
+
+using namespace fnpu;
+
+extern "C" {
+
+const char *fnpu_status_str(int s) {
+    switch (s) {
+        case FNPU_OK: return "ok";
+        case FNPU_EINVAL: return "invalid argument";
+        case FNPU_EUNSUPPORTED: return "unsupported shape";
+        case FNPU_ECUDA: return "CUDA runtime error";
+        case FNPU_EDEVICE_TIMEOUT: return "device-side wait timed out";
+        case FNPU_ENOMEM: return "out of memory";
+        case FNPU_EDEVICE_RANGE: return "device met an out-of-range slot";
+        default: return "unknown status";
+    }
+}
+
+int fnpu_version(void) { return 100; }
+
+int fnpu_kv_append(const fnpu_attn_desc *desc, const void *k_new, const void *v_new,
+                   const int64_t *slot_mapping, int32_t num_tokens, void *k_cache, void *v_cache,
+                   void *stream) {
+    int st;
+    if (!shape_ok(desc, &st)) return st;
+    if (num_tokens < 0) return FNPU_EINVAL;
+    if (num_tokens == 0) return FNPU_OK;
+    const bool latent = desc->v_in_k_latent != 0;
+    if (!k_new || !slot_mapping || !k_cache) return FNPU_EINVAL;
+    if (!latent && (!v_new || !v_cache)) return FNPU_EINVAL;
+    const uintptr_t mis = reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(k_cache) |
+                          (latent ? 0 : (reinterpret_cast<uintptr_t>(v_new) |
+                                         reinterpret_cast<uintptr_t>(v_cache)));
+    if (mis & 15u) return FNPU_EINVAL;
+    if (reinterpret_cast<uintptr_t>(slot_mapping) & 7u) return FNPU_EINVAL;
+    return launch_kv_append(desc, k_new, v_new, slot_mapping, num_tokens, k_cache, v_cache, stream);
+}
+
+int fnpu_check(void *stream) {
+    int flag = 0;
+    const int rc = read_and_clear_global_error(stream, &flag);
+    if (rc != FNPU_OK) return rc;
+    return flag ? FNPU_EDEVICE_RANGE : FNPU_OK;
+}
+
+int fnpu_mixed_attn_plan(const fnpu_attn_desc *desc, int32_t num_seqs, const int32_t *query_len,
+                         const int32_t *context_len, const uint8_t *phase,
+                         const int32_t *block_table, int32_t block_table_stride, void *stream,
+                         fnpu_plan **out) {
+    return fnpu_mixed_attn_plan_ex(desc, num_seqs, query_len, context_len, phase, block_table,
+                                   block_table_stride, nullptr, stream, out);
+}
+
+int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const int32_t *query_len,
+                            const int32_t *context_len, const uint8_t *phase,
+                            const int32_t *block_table, int32_t block_table_stride,
+                            const fnpu_plan_opts *opts, void *stream, fnpu_plan **out) {
+    int st;
+    if (!out) return FNPU_EINVAL;
+    if (!shape_ok(desc, &st)) return st;
+    if (num_seqs < 0) return FNPU_EINVAL;
+    if (num_seqs > 0 && (!query_len || !context_len || !phase || !block_table)) return FNPU_EINVAL;
+    fnpu_plan_opts o = {};
+    if (opts) o = *opts;
+    if (o.decode_split_keys < 0 || o.decode_share_pct < 0 || o.decode_share_pct > 100 || o.num_sms < 0)
+        return FNPU_EINVAL;
+    const int32_t bs = desc->block_size;
+
+    // validate the per-sequence metadata
+    int64_t T = 0;
+    int32_t width = 1;
+    bool has_decode = false, has_prefill = false;
+    for (int32_t s = 0; s < num_seqs; ++s) {
+        const int32_t q = query_len[s], c = context_len[s];
+        if (q < 1 || c < q) return FNPU_EINVAL;
+        if (phase[s] > 1) return FNPU_EINVAL;
+        if (phase[s] == 1 && q != 1) return FNPU_EINVAL;
+        has_decode |= phase[s] == 1;
+        has_prefill |= phase[s] == 0;
+        const int32_t nb = (c + bs - 1) / bs;
+        if (nb > block_table_stride) return FNPU_EINVAL;
+        for (int32_t j = 0; j < nb; ++j) {
+            const int32_t b = block_table[static_cast<int64_t>(s) * block_table_stride + j];
+            if (b < 0 || b >= desc->num_blocks) return FNPU_EINVAL;
+        }
+        width = std::max(width, nb);
+        T += q;
+    }
+    if (T > INT32_MAX) return FNPU_EINVAL;
+    if (num_seqs > 0) {
+        const int ks = kernel_support(desc, has_decode);
+        if (ks != FNPU_OK) return ks;
+    }
+    (void)has_prefill;
+
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return FNPU_ECUDA;
+    int sms = o.num_sms;
+    if (sms == 0 && cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return FNPU_ECUDA;
+
+    fnpu_plan *pl = new (std::nothrow) fnpu_plan();
+    if (!pl) return FNPU_ENOMEM;
+    pl->desc = *desc;
+    pl->scale = desc->softmax_scale > 0.f ? desc->softmax_scale
+                                          : static_cast<float>(1.0 / sqrt(static_cast<double>(desc->head_dim_qk)));
+    pl->num_seqs = num_seqs;
+    pl->num_tokens = T;
+    pl->bt_width = width;
+    pl->num_sms = sms;
+    pl->flags = o.flags;
+
+    const int32_t G = desc->num_q_heads / desc->num_kv_heads;
+    std::vector<SeqInfo> seqs(num_seqs);
+    std::vector<DecodeItem> ditems;
+    std::vector<PrefillItem> pitems;
+    std::vector<std::pair<int64_t, int32_t>> pcost;  // (cost, index) for LPT order
+
+    // decode split length: about 4 waves of 2 CTAs per SM over the decode keys
+    int64_t dec_keys = 0;
+    for (int32_t s = 0; s < num_seqs; ++s)
+        if (phase[s] == 1) dec_keys += static_cast<int64_t>(context_len[s]) * desc->num_kv_heads;
+    int32_t split = o.decode_split_keys;
+    if (split == 0) {
+        const int64_t target = 8LL * sms;
+        int64_t sk = (dec_keys + target - 1) / std::max<int64_t>(target, 1);
+        sk = (sk + 63) / 64 * 64;
+        split = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(sk, 256), 4096));
+    }
+
+    int32_t qs = 0, parts = 0, groups = 0;
+    for (int32_t s = 0; s < num_seqs; ++s) {
+        seqs[s] = SeqInfo{qs, query_len[s], context_len[s], s};
+        const int32_t q = query_len[s], c = context_len[s];
+        if (phase[s] == 1) {
+            const int32_t ns = (c + split - 1) / split;
+            for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh) {
+                const int32_t grp = groups++;
+                const int32_t base = ns > 1 ? parts : 0;
+                if (ns > 1) parts += ns;
+                for (int32_t sp = 0; sp < ns; ++sp) {
+                    const int32_t kb = sp * split, ke = std::min(c, kb + split);
+                    ditems.push_back(DecodeItem{s, kvh, kb, ke, sp, ns, base, grp});
+                }
+            }
+        } else {
+            const int32_t prefix = c - q;
+            for (int32_t r0 = 0; r0 < q; r0 += 64) {
+                const int32_t rows = std::min(64, q - r0);
+                for (int32_t h = 0; h < desc->num_q_heads; ++h) {
+                    pcost.emplace_back(static_cast<int64_t>(prefix) + r0 + rows,
+                                       static_cast<int32_t>(pitems.size()));
+                    pitems.push_back(PrefillItem{s, h, r0, rows});
+                }
+            }
+        }
+        qs += query_len[s];
+    }
+    // longest prefill tiles first; decode items longest first as well
+    std::stable_sort(pcost.begin(), pcost.end(),
+                     [](const std::pair<int64_t, int32_t> &a, const std::pair<int64_t, int32_t> &b) {
+                         return a.first > b.first;
+                     });
+    std::vector<PrefillItem> pordered;
+    pordered.reserve(pitems.size());
+    for (auto &pc : pcost) pordered.push_back(pitems[pc.second]);
+    std::stable_sort(ditems.begin(), ditems.end(), [](const DecodeItem &a, const DecodeItem &b) {
+        return (a.key_end - a.key_begin) > (b.key_end - b.key_begin);
+    });
+
+    pl->num_ditems = static_cast<int32_t>(ditems.size());
+    pl->num_pitems = static_cast<int32_t>(pordered.size());
+    pl->num_groups = groups;
+    pl->num_parts = parts;
+
+    // workspace: metadata (uploaded) then scratch (never read before written)
+    size_t off = 0;
+    const size_t o_seqs = off; off = align_up(off + sizeof(SeqInfo) * std::max(num_seqs, 1), 256);
+    const size_t o_bt = off; off = align_up(off + sizeof(int32_t) * static_cast<size_t>(std::max(num_seqs, 1)) * width, 256);
+    const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
+    const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
+    const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
+    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 4, 256);
+    const size_t meta_bytes = off;
+    const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * G, 256);
+    const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * G * desc->head_dim_v, 256);
+    pl->ws_bytes = off;
+
+    if (cudaMalloc(&pl->d_ws, pl->ws_bytes) != cudaSuccess) {
+        cudaGetLastError();
+        delete pl;
+        return FNPU_ENOMEM;
+    }
+    if (cudaMallocHost(&pl->h_stage, meta_bytes) != cudaSuccess) {
+        cudaGetLastError();
+        cudaFree(pl->d_ws);
+        delete pl;
+        return FNPU_ENOMEM;
+    }
+    uint8_t *h = static_cast<uint8_t *>(pl->h_stage);
+    memset(h, 0, meta_bytes);
+    if (num_seqs) memcpy(h + o_seqs, seqs.data(), sizeof(SeqInfo) * num_seqs);
+    for (int32_t s = 0; s < num_seqs; ++s)
+        memcpy(h + o_bt + sizeof(int32_t) * static_cast<size_t>(s) * width,
+               block_table + static_cast<int64_t>(s) * block_table_stride,
+               sizeof(int32_t) * static_cast<size_t>((context_len[s] + bs - 1) / bs));
+    if (!ditems.empty()) memcpy(h + o_di, ditems.data(), sizeof(DecodeItem) * ditems.size());
+    if (!pordered.empty()) memcpy(h + o_pi, pordered.data(), sizeof(PrefillItem) * pordered.size());
+
+    uint8_t *d = static_cast<uint8_t *>(pl->d_ws);
+    pl->d_seqs = reinterpret_cast<SeqInfo *>(d + o_seqs);
+    pl->d_bt = reinterpret_cast<int32_t *>(d + o_bt);
+    pl->d_ditems = reinterpret_cast<DecodeItem *>(d + o_di);
+    pl->d_pitems = reinterpret_cast<PrefillItem *>(d + o_pi);
+    pl->d_counters = reinterpret_cast<int32_t *>(d + o_cnt);
+    pl->d_err = reinterpret_cast<int32_t *>(d + o_err);
+    pl->d_part_lse = reinterpret_cast<float *>(d + o_plse);
+    pl->d_part_o = reinterpret_cast<float *>(d + o_po);
+    if (cudaMemcpyAsync(pl->d_ws, pl->h_stage, meta_bytes, cudaMemcpyHostToDevice,
+                        static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+        cudaGetLastError();
+        cudaFreeHost(pl->h_stage);
+        cudaFree(pl->d_ws);
+        delete pl;
+        return FNPU_ECUDA;
+    }
+    *out = pl;
+    return FNPU_OK;
+}
+
+int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache, const void *v_cache,
+                        void *out, float *lse, void *stream) {
+    if (!pl) return FNPU_EINVAL;
+    if (pl->num_tokens == 0) return FNPU_OK;
+    const bool latent = pl->desc.v_in_k_latent != 0;
+    if (!q || !k_cache || !out || !lse || (!latent && !v_cache)) return FNPU_EINVAL;
+    const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_cache) |
+                          reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(lse) |
+                          (latent ? 0 : reinterpret_cast<uintptr_t>(v_cache));
+    if (mis & 15u) return FNPU_EINVAL;
+
+    AttnParams p = {};
+    const fnpu_attn_desc &d = pl->desc;
+    p.q = q;
+    p.k_cache = k_cache;
+    p.v_cache = latent ? k_cache : v_cache;
+    p.out = out;
+    p.lse = lse;
+    p.seqs = pl->d_seqs;
+    p.block_table = pl->d_bt;
+    p.bt_stride = pl->bt_width;
+    p.num_q_heads = d.num_q_heads;
+    p.num_kv_heads = d.num_kv_heads;
+    p.group = d.num_q_heads / d.num_kv_heads;
+    p.block_size = d.block_size;
+    p.head_dim_qk = d.head_dim_qk;
+    p.head_dim_v = d.head_dim_v;
+    p.k_slot_stride = latent ? d.head_dim_qk : static_cast<int64_t>(d.num_kv_heads) * d.head_dim_qk;
+    p.v_slot_stride = latent ? d.head_dim_qk : static_cast<int64_t>(d.num_kv_heads) * d.head_dim_v;
+    p.scale_log2 = pl->scale * 1.4426950408889634f;
+    p.ditems = pl->d_ditems;
+    p.num_ditems = pl->num_ditems;
+    p.part_o = pl->d_part_o;
+    p.part_lse = pl->d_part_lse;
+    p.counters = pl->d_counters;
+    p.pitems = pl->d_pitems;
+    p.num_pitems = pl->num_pitems;
+    p.err = pl->d_err;
+
+    int rc = launch_decode_mma(p, stream);
+    if (rc != FNPU_OK) return rc;
+    rc = launch_prefill_mma(p, stream);
+    return rc;
+}
+
+int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
+    if (!pl) return FNPU_EINVAL;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FNPU_ECUDA;
+    int32_t v = 0;
+    if (cudaMemcpy(&v, pl->d_err, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return FNPU_ECUDA;
+    if (v != 0) {
+        const int32_t zero = 0;
+        if (cudaMemcpy(pl->d_err, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+            return FNPU_ECUDA;
+        return FNPU_EDEVICE_TIMEOUT;
+    }
+    return FNPU_OK;
+}
+
+void fnpu_plan_destroy(fnpu_plan *pl) {
+    if (!pl) return;
+    cudaDeviceSynchronize();
+    if (pl->h_stage) cudaFreeHost(pl->h_stage);
+    if (pl->d_ws) cudaFree(pl->d_ws);
+    delete pl;
+}
+
+int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_items,
+                   int32_t *launches_per_run, int64_t *workspace_bytes) {
+    if (!pl) return FNPU_EINVAL;
+    if (prefill_items) *prefill_items = pl->num_pitems;
+    if (decode_items) *decode_items = pl->num_ditems;
+    if (launches_per_run) *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0);
+    if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_bytes);
+    return FNPU_OK;
+}
+
+}  // extern "C"

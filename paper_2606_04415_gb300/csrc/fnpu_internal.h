@@ -1,0 +1,71 @@
+// Internal structures shared between the host planner and the kernels.
+#pragma once
+
+#include <stdint.h>
+
+#include "../../include/fnpu.h"
+
+namespace fnpu {
+
+// One decode split item: keys [key_begin, key_end) of sequence `seq` for kv
+// head `kvh`, all G query heads of that group at the sequence's single query
+// position. Splits of one (seq, kvh) group share `group` (their merge counter)
+// and write partial results to scratch rows part_base + split.
+struct DecodeItem {
+    int32_t seq, kvh, key_begin, key_end;
+    int32_t split, num_splits, part_base, group;
+};
+static_assert(sizeof(DecodeItem) == 32, "DecodeItem layout");
+
+// One prefill tile: query rows [row_begin, row_begin + rows) of sequence
+// `seq`'s chunk for query head `head` (the mma.sync path) or for kv head
+// `head` with all its query heads packed (the tcgen05 path).
+struct PrefillItem {
+    int32_t seq, head, row_begin, rows;
+};
+static_assert(sizeof(PrefillItem) == 16, "PrefillItem layout");
+
+// Per-sequence metadata on the device.
+struct SeqInfo {
+    int32_t q_start;  // first query token of the sequence in q/out/lse
+    int32_t q_len;
+    int32_t ctx_len;  // includes this step's q_len new tokens
+    int32_t bt_row;   // row of the sequence in the device block table
+};
+static_assert(sizeof(SeqInfo) == 16, "SeqInfo layout");
+
+struct AttnParams {
+    const void *q;        // bf16 [T, Hq, dqk]
+    const void *k_cache;  // bf16 [nb, bs, Hkv, dqk] (latent: [nb, bs, dqk])
+    const void *v_cache;  // bf16 [nb, bs, Hkv, dv]  (latent: == k_cache)
+    void *out;            // bf16 [T, Hq, dv]
+    float *lse;           // fp32 [T, Hq]
+    const SeqInfo *seqs;
+    const int32_t *block_table;  // [num_seqs, bt_stride]
+    int32_t bt_stride;
+    int32_t num_q_heads, num_kv_heads, group, block_size;
+    int32_t head_dim_qk, head_dim_v;
+    int64_t k_slot_stride;  // elements between consecutive slots of k_cache
+    int64_t v_slot_stride;
+    float scale_log2;       // softmax scale * log2(e)
+    // decode split-KV
+    const DecodeItem *ditems;
+    int32_t num_ditems;
+    float *part_o;          // fp32 [num_parts, group, dv]
+    float *part_lse;        // fp32 [num_parts, group] (log2 domain)
+    int32_t *counters;      // [num_groups], zero between runs
+    // prefill
+    const PrefillItem *pitems;
+    int32_t num_pitems;
+    int32_t *err;           // device error flag of the plan
+};
+
+// Launchers (defined in the .cu files).
+int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_new,
+                     const int64_t *slots, int32_t num_tokens, void *k_cache, void *v_cache,
+                     void *stream);
+int read_and_clear_global_error(void *stream, int *flag);
+int launch_decode_mma(const AttnParams &p, void *stream);
+int launch_prefill_mma(const AttnParams &p, void *stream);
+
+}  // namespace fnpu

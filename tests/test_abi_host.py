@@ -1,0 +1,112 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds, loads
+and exports every entry point declared in include/fnpu.h, and argument
+validation rejects bad metadata before any CUDA call is made."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2606_04415_gb300 as fnpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_symbols():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(fnpu_[a-z_0-9]+)\s*\(", src))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = fnpu.load()
+    declared = _declared_symbols()
+    assert declared, "no declarations found"
+    assert declared == set(fnpu.EXPORTED)
+    for name in declared:
+        assert hasattr(lib, name), name
+
+
+def test_status_strings_and_version():
+    assert fnpu.status_str(fnpu.FNPU_OK) == "ok"
+    assert "invalid" in fnpu.status_str(fnpu.FNPU_EINVAL)
+    assert fnpu.status_str(12345) == "unknown status"
+    assert fnpu.version() >= 100
+
+
+def _plan_rc(desc, ql, cl, ph, bt, opts=None):
+    lib = fnpu.load()
+    ql = np.ascontiguousarray(ql, np.int32)
+    cl = np.ascontiguousarray(cl, np.int32)
+    ph = np.ascontiguousarray(ph, np.uint8)
+    bt = np.ascontiguousarray(bt, np.int32)
+    out = ctypes.c_void_p()
+    return lib.fnpu_mixed_attn_plan_ex(ctypes.byref(desc), len(ql), ql.ctypes.data, cl.ctypes.data,
+                                       ph.ctypes.data, bt.ctypes.data, bt.shape[1],
+                                       None if opts is None else ctypes.byref(opts), None,
+                                       ctypes.byref(out))
+
+
+QWEN = dict(num_q_heads=28, num_kv_heads=4, head_dim_qk=128, head_dim_v=128, block_size=16,
+            num_blocks=100)
+
+
+@pytest.mark.parametrize("case", [
+    "ctx_lt_q", "q_zero", "decode_q2", "phase_2", "block_oob", "block_neg", "stride_short",
+])
+def test_plan_rejects_bad_metadata(case):
+    desc = fnpu.make_desc(**QWEN)
+    ql, cl, ph = [4, 1], [10, 40], [0, 1]
+    bt = np.zeros((2, 4), np.int32)
+    if case == "ctx_lt_q":
+        cl = [3, 40]
+    elif case == "q_zero":
+        ql = [0, 1]
+    elif case == "decode_q2":
+        ql = [4, 2]
+    elif case == "phase_2":
+        ph = [0, 2]
+    elif case == "block_oob":
+        bt[1, 2] = 100
+    elif case == "block_neg":
+        bt[0, 0] = -1
+    elif case == "stride_short":
+        bt = np.zeros((2, 2), np.int32)
+    assert _plan_rc(desc, ql, cl, ph, bt) == fnpu.FNPU_EINVAL
+
+
+def test_plan_rejects_bad_shape_and_options():
+    bt = np.zeros((1, 4), np.int32)
+    bad = fnpu.make_desc(**dict(QWEN, num_q_heads=30))  # not a multiple of Hkv
+    assert _plan_rc(bad, [1], [5], [1], bt) == fnpu.FNPU_EINVAL
+    bad = fnpu.make_desc(**dict(QWEN, block_size=0))
+    assert _plan_rc(bad, [1], [5], [1], bt) == fnpu.FNPU_EINVAL
+    opts = fnpu.PlanOpts(-5, 0, 0, 0)
+    assert _plan_rc(fnpu.make_desc(**QWEN), [1], [5], [1], bt, opts) == fnpu.FNPU_EINVAL
+    opts = fnpu.PlanOpts(0, 101, 0, 0)
+    assert _plan_rc(fnpu.make_desc(**QWEN), [1], [5], [1], bt, opts) == fnpu.FNPU_EINVAL
+
+
+def test_plan_reports_unsupported_head_dims():
+    bt = np.zeros((1, 4), np.int32)
+    desc = fnpu.make_desc(**dict(QWEN, head_dim_qk=96, head_dim_v=96))
+    assert _plan_rc(desc, [1], [5], [1], bt) == fnpu.FNPU_EUNSUPPORTED
+
+
+def test_append_and_run_reject_null_pointers():
+    lib = fnpu.load()
+    desc = fnpu.make_desc(**QWEN)
+    rc = lib.fnpu_kv_append(ctypes.byref(desc), None, None, None, 4, None, None, None)
+    assert rc == fnpu.FNPU_EINVAL
+    rc = lib.fnpu_kv_append(ctypes.byref(desc), 16, 32, 64, -1, 128, 256, None)
+    assert rc == fnpu.FNPU_EINVAL
+    rc = lib.fnpu_kv_append(ctypes.byref(desc), 17, 32, 64, 4, 128, 256, None)  # misaligned
+    assert rc == fnpu.FNPU_EINVAL
+    assert lib.fnpu_mixed_attn_run(None, None, None, None, None, None, None) == fnpu.FNPU_EINVAL
+    assert lib.fnpu_plan_check(None, None) == fnpu.FNPU_EINVAL
+    lib.fnpu_plan_destroy(None)  # ignored

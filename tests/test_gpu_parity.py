@@ -1,0 +1,225 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Tolerances: |O - O_ref| <= 2e-2 and |LSE - LSE_ref| <= 1e-3 (bf16 inputs,
+fp32 scores and accumulation, bf16 output); KV append bit-exact over the
+whole pool, untouched (canary) slots included.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import workloads as W
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+O_TOL = 2e-2
+LSE_TOL = 1e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2606_04415_gb300 as fnpu
+    fnpu.load()
+
+
+def _step(batch, **opts):
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    o = fnpu.PlanOpts(opts.get("split", 0), opts.get("share", 0), opts.get("sms", 0),
+                      opts.get("flags", 0))
+    st = DeviceStep(batch, opts=o)
+    st.run()
+    return st
+
+
+def _compare(batch, out, lse, tokens=None, kc=None, vc=None):
+    if kc is None:
+        ref_o, ref_l, _, _ = oracle.run_step(batch, tokens=tokens)
+    else:
+        sh = batch.shape
+        ref_o, ref_l = oracle.attention(batch.query_len, batch.context_len, batch.block_table,
+                                        batch.q, kc, vc, num_q_heads=sh.num_q_heads,
+                                        num_kv_heads=sh.num_kv_heads, head_dim_qk=sh.head_dim_qk,
+                                        head_dim_v=sh.head_dim_v, block_size=sh.block_size,
+                                        latent=sh.latent, tokens=tokens)
+    if tokens is not None:
+        out, lse = out[tokens], lse[tokens]
+    assert np.isfinite(out).all() and np.isfinite(lse).all()
+    eo = np.abs(out - ref_o).max()
+    el = np.abs(lse - ref_l).max()
+    assert eo <= O_TOL, f"max |dO| = {eo}"
+    assert el <= LSE_TOL, f"max |dLSE| = {el}"
+    return eo, el
+
+
+def _sample_tokens(batch, per_seq_rows=6, seed=0):
+    """Rows the oracle recomputes at full size: every decode row, and for each
+    prefill chunk its first/last rows, tile boundaries and random rows."""
+    rng = np.random.default_rng(seed)
+    qs = batch.query_start
+    toks = []
+    for s in range(batch.num_seqs):
+        q = int(batch.query_len[s])
+        if q == 1:
+            toks.append(qs[s])
+            continue
+        rows = {0, q - 1, min(63, q - 1), min(64, q - 1), min(127, q - 1), min(128, q - 1)}
+        rows |= set(rng.integers(0, q, size=per_seq_rows).tolist())
+        toks += [qs[s] + r for r in sorted(rows)]
+    return np.asarray(sorted(set(toks)), np.int64)
+
+
+def test_kv_append_bit_exact_whole_pool():
+    batch = W.make_batch("tiny", seed=1)
+    st = _step(batch)
+    kc, vc = st.cache_bits()
+    ref_k = oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping)
+    ref_v = oracle.kv_append(batch.v_cache, batch.v_new, batch.slot_mapping)
+    assert np.array_equal(kc, ref_k) and np.array_equal(vc, ref_v)
+
+
+def test_kv_append_padding_and_range_flag():
+    import paper_2606_04415_gb300 as fnpu
+    batch = W.make_batch("tiny", seed=2)
+    st = _step(batch)
+    assert fnpu.check() == fnpu.FNPU_OK
+    # padding slots (-1) are skipped; an out-of-range slot is skipped and flagged
+    slots = batch.slot_mapping.copy()
+    slots[::7] = -1
+    nslot = batch.num_blocks * batch.shape.block_size
+    slots[5] = nslot + 3
+    k0 = st.k_cache.clone()
+    v0 = st.v_cache.clone()
+    sm = torch.from_numpy(slots).cuda()
+    fnpu.kv_append(st.desc, st.k_new, st.v_new, sm, st.k_cache, st.v_cache)
+    assert fnpu.check() == fnpu.FNPU_EDEVICE_RANGE
+    assert fnpu.check() == fnpu.FNPU_OK  # cleared
+    good = slots.copy()
+    good[5] = -1
+    ref_k = oracle.kv_append(k0.view(torch.int16).cpu().numpy().view(np.uint16), batch.k_new, good)
+    ref_v = oracle.kv_append(v0.view(torch.int16).cpu().numpy().view(np.uint16), batch.v_new, good)
+    kc, vc = st.cache_bits()
+    assert np.array_equal(kc, ref_k) and np.array_equal(vc, ref_v)
+
+
+def test_kv_append_full_size_bit_exact():
+    batch = W.make_batch("qwen_coloc", seed=0)
+    st = _step(batch)
+    kc, vc = st.cache_bits()
+    assert np.array_equal(kc, oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping))
+    assert np.array_equal(vc, oracle.kv_append(batch.v_cache, batch.v_new, batch.slot_mapping))
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_tiny_mixed_batch_all_rows(seed):
+    batch = W.make_batch("tiny", seed=seed)
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+@pytest.mark.parametrize("split", [64, 128, 4096])
+def test_decode_split_counts_agree(split):
+    batch = W.make_batch("tiny", seed=5)
+    st = _step(batch, split=split)
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_plan_reuse_runs_repeatedly():
+    batch = W.make_batch("tiny", seed=6)
+    st = _step(batch, split=64)
+    out1, lse1 = st.results()
+    for _ in range(3):
+        st.run()
+    out2, lse2 = st.results()
+    assert np.array_equal(out1, out2) and np.array_equal(lse1, lse2)
+
+
+def test_qwen_decode_full_size_all_rows():
+    batch = W.make_batch("qwen_decode", seed=0)
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_qwen_prefill_full_size_sampled_rows():
+    batch = W.make_batch("qwen_prefill", seed=0)
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse, tokens=_sample_tokens(batch))
+
+
+def test_qwen_coloc_full_size_sampled_rows():
+    batch = W.make_batch("qwen_coloc", seed=0)
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse, tokens=_sample_tokens(batch, per_seq_rows=10))
+
+
+@pytest.mark.parametrize("bs", [1, 16, 32])
+@pytest.mark.parametrize("dim", [64, 128])
+def test_ragged_edges(bs, dim):
+    """ctx = 1 prefill, 1-row and ragged chunks, prefixes not on block edges."""
+    sh = W.Shape(8, 2, dim, dim, bs, False)
+    ql = [1, 1, 63, 65, 130, 1, 1, 7]
+    ctx = [1, 37, 63, 100, 131, 1, 2, 7 + 91]
+    ph = [0, 1, 0, 0, 0, 1, 1, 0]
+    rng = np.random.default_rng(bs * 1000 + dim)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="ragged")
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_block_permutation_invariance_gpu():
+    batch = W.make_batch("tiny", seed=7)
+    st = _step(batch)
+    out, lse = st.results()
+    perm = np.random.default_rng(3).permutation(batch.num_blocks)
+    kc = np.empty_like(batch.k_cache)
+    vc = np.empty_like(batch.v_cache)
+    kc[perm] = batch.k_cache
+    vc[perm] = batch.v_cache
+    b2 = W.Batch(**{**batch.__dict__, "k_cache": kc, "v_cache": vc,
+                    "block_table": perm[batch.block_table].astype(np.int32),
+                    "slot_mapping": (perm[batch.slot_mapping // 16] * 16 + batch.slot_mapping % 16)})
+    st2 = _step(b2)
+    out2, lse2 = st2.results()
+    assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
+
+
+def test_decode_row_matches_prefill_row_gpu():
+    """Decode of position t (decode kernel) vs row t of a prefill (prefill kernel)."""
+    sh = W.SHAPES["qwen"]
+    L = 300
+    rng = np.random.default_rng(21)
+    pre = W.build_batch(sh, [L], [L], [0], rng, name="pre", extra_bt_cols=0)
+    st = _step(pre)
+    out_p, lse_p = st.results()
+    kc, vc = st.cache_bits()
+    positions = [0, 15, 16, 150, 299]
+    dec = W.Batch(name="dec", shape=sh, seed=0, query_len=np.ones(len(positions), np.int32),
+                  context_len=np.asarray([p + 1 for p in positions], np.int32),
+                  phase=np.ones(len(positions), np.uint8),
+                  block_table=np.repeat(pre.block_table, len(positions), 0), num_blocks=pre.num_blocks,
+                  q=pre.q[positions], k_new=pre.k_new[positions], v_new=pre.v_new[positions],
+                  slot_mapping=pre.slot_mapping[positions], k_cache=kc, v_cache=vc)
+    st2 = _step(dec)
+    out_d, lse_d = st2.results()
+    assert np.abs(out_d - out_p[positions]).max() <= O_TOL
+    assert np.abs(lse_d - lse_p[positions]).max() <= LSE_TOL
+
+
+def test_empty_batch_is_a_noop():
+    import paper_2606_04415_gb300 as fnpu
+    desc = fnpu.make_desc(4, 2, 64, 64, 16, 8)
+    plan = fnpu.mixed_attn_plan(desc, np.zeros(0, np.int32), np.zeros(0, np.int32),
+                                np.zeros(0, np.uint8), np.zeros((0, 1), np.int32))
+    dummy = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
+    fnpu.mixed_attn_run(plan, dummy, dummy, dummy, dummy, dummy.float())
+    assert fnpu.plan_check(plan) == fnpu.FNPU_OK
+    assert plan.info()["prefill_items"] == 0 and plan.info()["decode_items"] == 0
