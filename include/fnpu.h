@@ -159,6 +159,49 @@ void fnpu_plan_destroy(fnpu_plan *plan);
 int fnpu_plan_info(const fnpu_plan *plan, int32_t *prefill_items, int32_t *decode_items,
                    int32_t *launches_per_run, int64_t *workspace_bytes);
 
+/*
+ * Decode attention without any allocation. The paper has no counterpart:
+ * this entry point exists for callers that may not call cudaMalloc at all,
+ * for instance code that must stay inside memory another framework reserved
+ * up front, or a serving process whose device memory is fixed once at start.
+ * A plan cannot serve them, because fnpu_mixed_attn_plan allocates a device
+ * workspace. This call computes the same GQA-packed split-KV decode as the
+ * decode items of fnpu_mixed_attn_run, but keeps its split scratch (partial
+ * outputs, partial log-sum-exps, merge counters) in one fixed array of
+ * FNPU_NOALLOC_SCRATCH_BYTES inside the library, which every GPU that loads
+ * the library holds until the process exits. It calls no cudaMalloc, no
+ * cudaFree and no allocating library routine.
+ *
+ * Every sequence is a decode: query_len = 1, and sequence s's query is row s.
+ *   context_len   device int32 [num_seqs], each in [1, max_context_len]
+ *                 (counts the new token)
+ *   block_table   device int32 [num_seqs, block_table_stride], stride >=
+ *                 ceil(max_context_len / block_size)
+ *   max_context_len  host bound on context_len; it sizes the grid
+ *   split_keys    keys per split, a multiple of 64; 0 selects 512
+ *   q             device bf16 [num_seqs, Hq, d]; out bf16 [num_seqs, Hq, d];
+ *                 lse fp32 [num_seqs, Hq]; k_cache / v_cache as above
+ * Supports split K/V caches with d_qk = d_v in {64, 128} and Hq/Hkv <= 8.
+ * Errors: FNPU_EINVAL for bad arguments and for requests whose scratch
+ * (4 B per counter, plus 4 B * (Hq/Hkv) * (d + 1) per split, for
+ * num_seqs * Hkv * ceil(max_context_len / split_keys) splits) exceeds
+ * FNPU_NOALLOC_SCRATCH_BYTES; FNPU_EUNSUPPORTED for other shapes;
+ * FNPU_ECUDA. Nothing is launched on error.
+ * The first call on a device looks up the scratch array's device address
+ * (cudaGetSymbolAddress) while that device is current; make that first call
+ * before any stream capture. All calls share the one array, which keeps the
+ * last call's contents; each call clears its merge counters itself with
+ * cudaMemsetAsync on `stream`. Calls that overlap on the GPU (on different
+ * streams, or with no ordering between them) race on the array and must not
+ * be issued.
+ */
+#define FNPU_NOALLOC_SCRATCH_BYTES (16u << 20)
+int fnpu_decode_attn_noalloc(const fnpu_attn_desc *desc, int32_t num_seqs,
+                             const int32_t *context_len, const int32_t *block_table,
+                             int32_t block_table_stride, int32_t max_context_len,
+                             int32_t split_keys, const void *q, const void *k_cache,
+                             const void *v_cache, void *out, float *lse, void *stream);
+
 /* Static description of a status code; never NULL. */
 const char *fnpu_status_str(int status);
 

@@ -38,7 +38,7 @@ PLAN_NO_TCGEN05 = 2
 EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
-    "fnpu_version",
+    "fnpu_version", "fnpu_decode_attn_noalloc",
 )
 
 
@@ -90,11 +90,13 @@ def load(build_if_missing: bool = True):
     lib.fnpu_plan_destroy.restype = None
     lib.fnpu_plan_info.argtypes = [P, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32),
                                    ctypes.POINTER(i64)]
+    lib.fnpu_decode_attn_noalloc.argtypes = [ctypes.POINTER(AttnDesc), i32, P, P, i32, i32, i32,
+                                             P, P, P, P, P, P]
     lib.fnpu_status_str.argtypes = [ctypes.c_int]
     lib.fnpu_status_str.restype = ctypes.c_char_p
     for name in ("fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex",
                  "fnpu_mixed_attn_run", "fnpu_plan_check", "fnpu_check", "fnpu_plan_info",
-                 "fnpu_version"):
+                 "fnpu_version", "fnpu_decode_attn_noalloc"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -204,6 +206,20 @@ def mixed_attn_run(plan: Plan, q, k_cache, v_cache, out, lse, stream=None) -> No
                                     _dptr(out), _dptr(lse), _stream(stream))
     if rc != FNPU_OK:
         raise FnpuError(rc, "fnpu_mixed_attn_run")
+
+
+def decode_attn_noalloc(desc: AttnDesc, context_len, block_table, max_context_len: int, q,
+                        k_cache, v_cache, out, lse, split_keys: int = 0, stream=None) -> None:
+    """Decode attention with the library's fixed scratch and no allocation
+    (``fnpu_decode_attn_noalloc``); context_len and block_table are device
+    int32 tensors."""
+    rc = load().fnpu_decode_attn_noalloc(ctypes.byref(desc), int(context_len.shape[0]),
+                                         _dptr(context_len), _dptr(block_table),
+                                         int(block_table.shape[1]), int(max_context_len),
+                                         int(split_keys), _dptr(q), _dptr(k_cache), _dptr(v_cache),
+                                         _dptr(out), _dptr(lse), _stream(stream))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_decode_attn_noalloc")
 
 
 def plan_check(plan: Plan, stream=None) -> int:
