@@ -26,6 +26,7 @@ struct fnpu_plan {
     int32_t bt_width = 0;
     int32_t num_sms = 0;
     int32_t flags = 0;
+    bool use_tc = false;
     int32_t num_ditems = 0, num_pitems = 0, num_groups = 0, num_parts = 0;
     void *d_ws = nullptr;
     size_t ws_bytes = 0;
@@ -182,6 +183,9 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->bt_width = width;
     pl->num_sms = sms;
     pl->flags = o.flags;
+    pl->use_tc = !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
+                 prefill_tc_supported(desc->head_dim_qk, desc->head_dim_v, bs,
+                                      desc->num_q_heads / desc->num_kv_heads);
 
     const int32_t G = desc->num_q_heads / desc->num_kv_heads;
     std::vector<SeqInfo> seqs(num_seqs);
@@ -214,6 +218,18 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 for (int32_t sp = 0; sp < ns; ++sp) {
                     const int32_t kb = sp * split, ke = std::min(c, kb + split);
                     ditems.push_back(DecodeItem{s, kvh, kb, ke, sp, ns, base, grp});
+                }
+            }
+        } else if (pl->use_tc) {
+            // tcgen05 tiles: P positions x G heads of one kv head per tile
+            const int32_t prefix = c - q;
+            const int32_t P = prefill_tc_rows_per_item(G);
+            for (int32_t r0 = 0; r0 < q; r0 += P) {
+                const int32_t rows = std::min(P, q - r0);
+                for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh) {
+                    pcost.emplace_back(static_cast<int64_t>(prefix) + r0 + rows,
+                                       static_cast<int32_t>(pitems.size()));
+                    pitems.push_back(PrefillItem{s, kvh, r0, rows});
                 }
             }
         } else {
@@ -326,6 +342,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.num_kv_heads = d.num_kv_heads;
     p.group = d.num_q_heads / d.num_kv_heads;
     p.block_size = d.block_size;
+    p.num_blocks = d.num_blocks;
     p.head_dim_qk = d.head_dim_qk;
     p.head_dim_v = d.head_dim_v;
     p.k_slot_stride = latent ? d.head_dim_qk : static_cast<int64_t>(d.num_kv_heads) * d.head_dim_qk;
@@ -342,8 +359,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
 
     int rc = launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
-    rc = launch_prefill_mma(p, stream);
-    return rc;
+    return pl->use_tc ? launch_prefill_tc(p, stream) : launch_prefill_mma(p, stream);
 }
 
 int fnpu_plan_check(const fnpu_plan *pl, void *stream) {

@@ -43,7 +43,7 @@ struct AttnParams {
     const SeqInfo *seqs;
     const int32_t *block_table;  // [num_seqs, bt_stride]
     int32_t bt_stride;
-    int32_t num_q_heads, num_kv_heads, group, block_size;
+    int32_t num_q_heads, num_kv_heads, group, block_size, num_blocks;
     int32_t head_dim_qk, head_dim_v;
     int64_t k_slot_stride;  // elements between consecutive slots of k_cache
     int64_t v_slot_stride;
@@ -67,5 +67,8 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
 int read_and_clear_global_error(void *stream, int *flag);
 int launch_decode_mma(const AttnParams &p, void *stream);
 int launch_prefill_mma(const AttnParams &p, void *stream);
+int launch_prefill_tc(const AttnParams &p, void *stream);
+bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
+int prefill_tc_rows_per_item(int group);
 
 }  // namespace fnpu

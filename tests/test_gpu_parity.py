@@ -32,6 +32,7 @@ def _step(batch, **opts):
                       opts.get("flags", 0))
     st = DeviceStep(batch, opts=o)
     st.run()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK, "device error flag raised"
     return st
 
 
@@ -113,10 +114,14 @@ def test_kv_append_full_size_bit_exact():
     assert np.array_equal(vc, oracle.kv_append(batch.v_cache, batch.v_new, batch.slot_mapping))
 
 
+NO_TC = 2  # FNPU_PLAN_NO_TCGEN05: prefill on the mma.sync path
+
+
+@pytest.mark.parametrize("flags", [0, NO_TC])
 @pytest.mark.parametrize("seed", [0, 1, 2])
-def test_tiny_mixed_batch_all_rows(seed):
+def test_tiny_mixed_batch_all_rows(seed, flags):
     batch = W.make_batch("tiny", seed=seed)
-    st = _step(batch)
+    st = _step(batch, flags=flags)
     out, lse = st.results()
     _compare(batch, out, lse)
 
@@ -146,9 +151,10 @@ def test_qwen_decode_full_size_all_rows():
     _compare(batch, out, lse)
 
 
-def test_qwen_prefill_full_size_sampled_rows():
+@pytest.mark.parametrize("flags", [0, NO_TC])
+def test_qwen_prefill_full_size_sampled_rows(flags):
     batch = W.make_batch("qwen_prefill", seed=0)
-    st = _step(batch)
+    st = _step(batch, flags=flags)
     out, lse = st.results()
     _compare(batch, out, lse, tokens=_sample_tokens(batch))
 
@@ -160,9 +166,10 @@ def test_qwen_coloc_full_size_sampled_rows():
     _compare(batch, out, lse, tokens=_sample_tokens(batch, per_seq_rows=10))
 
 
-@pytest.mark.parametrize("bs", [1, 16, 32])
+@pytest.mark.parametrize("flags", [0, NO_TC])
+@pytest.mark.parametrize("bs", [1, 16, 32, 64])
 @pytest.mark.parametrize("dim", [64, 128])
-def test_ragged_edges(bs, dim):
+def test_ragged_edges(bs, dim, flags):
     """ctx = 1 prefill, 1-row and ragged chunks, prefixes not on block edges."""
     sh = W.Shape(8, 2, dim, dim, bs, False)
     ql = [1, 1, 63, 65, 130, 1, 1, 7]
@@ -170,7 +177,7 @@ def test_ragged_edges(bs, dim):
     ph = [0, 1, 0, 0, 0, 1, 1, 0]
     rng = np.random.default_rng(bs * 1000 + dim)
     batch = W.build_batch(sh, ql, ctx, ph, rng, name="ragged")
-    st = _step(batch)
+    st = _step(batch, flags=flags)
     out, lse = st.results()
     _compare(batch, out, lse)
 
@@ -223,3 +230,21 @@ def test_empty_batch_is_a_noop():
     fnpu.mixed_attn_run(plan, dummy, dummy, dummy, dummy, dummy.float())
     assert fnpu.plan_check(plan) == fnpu.FNPU_OK
     assert plan.info()["prefill_items"] == 0 and plan.info()["decode_items"] == 0
+
+
+@pytest.mark.parametrize("group", [1, 3, 7, 8])
+def test_prefill_gqa_packing_groups(group):
+    """tcgen05 tiles pack floor(128 / G) positions x G heads; sweep G."""
+    sh = W.Shape(2 * group, 2, 128, 128, 16, False)
+    rng = np.random.default_rng(100 + group)
+    batch = W.build_batch(sh, [200, 37, 1], [200, 300, 50], [0, 0, 1], rng, name="gqa")
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_tc_and_mma_prefill_agree_on_coloc():
+    batch = W.make_batch("qwen_coloc", seed=2)
+    a = _step(batch).results()
+    b = _step(batch, flags=NO_TC).results()
+    assert np.abs(a[0] - b[0]).max() <= O_TOL and np.abs(a[1] - b[1]).max() <= LSE_TOL
