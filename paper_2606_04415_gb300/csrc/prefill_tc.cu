@@ -212,7 +212,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int P = kRows / G;
         const int pl = r / G, hl = r % G;
         const bool row_ok = (r < P * G) && (pl < it.rows);
+        // rows past the item (padding) keep a position too; their results are
+        // never stored, so they need no masking of their own
         const int pos = prefix + it.row_begin + pl;
+        const int min_pos = prefix + it.row_begin;
         const int64_t tok = si.q_start + it.row_begin + pl;
         const int head = kvh * G + hl;
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
@@ -245,15 +248,33 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc::tmem_ld32(lane_addr + kColS, *reinterpret_cast<uint32_t(*)[32]>(&s[0]));
             tc::tmem_ld32(lane_addr + kColS + 32, *reinterpret_cast<uint32_t(*)[32]>(&s[32]));
             tc::tmem_wait_ld();
+            // tiles that reach past the first row's position need the causal
+            // mask; all others are fully visible to every row of the item
             const int k0 = i * kKeys;
-            float tmax = -INFINITY;
+            const bool masked_tile = k0 + kKeys - 1 > min_pos;
+            float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+            if (masked_tile) {
 #pragma unroll
-            for (int j = 0; j < kKeys; ++j) {
-                float x = __uint_as_float(s[j]) * p.scale_log2;
-                x = row_ok ? ((k0 + j <= pos) ? x : -INFINITY) : 0.f;
-                s[j] = __float_as_uint(x);
-                tmax = fmaxf(tmax, x);
+                for (int j = 0; j < kKeys; j += 4) {
+                    float v0 = __uint_as_float(s[j]), v1 = __uint_as_float(s[j + 1]);
+                    float v2 = __uint_as_float(s[j + 2]), v3 = __uint_as_float(s[j + 3]);
+                    v0 = (k0 + j <= pos) ? v0 : -INFINITY;
+                    v1 = (k0 + j + 1 <= pos) ? v1 : -INFINITY;
+                    v2 = (k0 + j + 2 <= pos) ? v2 : -INFINITY;
+                    v3 = (k0 + j + 3 <= pos) ? v3 : -INFINITY;
+                    s[j] = __float_as_uint(v0); s[j + 1] = __float_as_uint(v1);
+                    s[j + 2] = __float_as_uint(v2); s[j + 3] = __float_as_uint(v3);
+                    mx0 = fmaxf(mx0, v0); mx1 = fmaxf(mx1, v1); mx2 = fmaxf(mx2, v2); mx3 = fmaxf(mx3, v3);
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < kKeys; j += 4) {
+                    mx0 = fmaxf(mx0, __uint_as_float(s[j])); mx1 = fmaxf(mx1, __uint_as_float(s[j + 1]));
+                    mx2 = fmaxf(mx2, __uint_as_float(s[j + 2])); mx3 = fmaxf(mx3, __uint_as_float(s[j + 3]));
+                }
             }
+            // the scale is positive, so the max of scaled scores is the scaled max
+            const float tmax = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * p.scale_log2;
             const bool need = (m_run == -INFINITY) ? (tmax != -INFINITY) : (tmax > m_run + kRescaleThreshold);
             if (__any_sync(0xffffffffu, need)) {
                 const float m_new = need ? fmaxf(m_run, tmax) : m_run;
@@ -272,15 +293,18 @@ __global__ void __launch_bounds__(kThreads, 2)
                 l *= alpha;
                 m_run = m_new;
             }
-            const float base = (m_run == -INFINITY) ? 0.f : m_run;
+            const float nbase = (m_run == -INFINITY) ? 0.f : -m_run;
+            const float sc = p.scale_log2;
+            float l0 = 0.f, l1 = 0.f;
             uint32_t pk[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
-                const float p0 = fast_exp2(__uint_as_float(s[2 * j]) - base);
-                const float p1 = fast_exp2(__uint_as_float(s[2 * j + 1]) - base);
-                l += p0 + p1;
+                const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * j]), sc, nbase));
+                const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * j + 1]), sc, nbase));
+                if (j & 1) l1 += p0 + p1; else l0 += p0 + p1;
                 pk[j] = pack_bf16x2(p0, p1);
             }
+            l += l0 + l1;
             tc::tmem_st32(lane_addr + kColS, pk);
             tc::tmem_wait_st();
             tc::fence_before_sync();
