@@ -205,6 +205,10 @@ int fnpu_decode_attn_noalloc(const fnpu_attn_desc *desc, int32_t num_seqs,
 /* Static description of a status code; never NULL. */
 const char *fnpu_status_str(int status);
 
+/* Text of the last failed CUDA call on this thread ("" if none), e.g. to
+ * explain an FNPU_ECUDA; never NULL, valid until the next library call. */
+const char *fnpu_last_cuda_error(void);
+
 /* Library version, major * 10000 + minor * 100 + patch. */
 int fnpu_version(void);
 

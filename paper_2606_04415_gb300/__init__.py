@@ -38,13 +38,16 @@ PLAN_NO_TCGEN05 = 2
 EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
-    "fnpu_version", "fnpu_decode_attn_noalloc",
+    "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error",
 )
 
 
 class FnpuError(RuntimeError):
     def __init__(self, code: int, what: str):
-        super().__init__(f"{what}: {status_str(code)} ({code})")
+        msg = f"{what}: {status_str(code)} ({code})"
+        if code == FNPU_ECUDA:
+            msg += f" [{last_cuda_error()}]"
+        super().__init__(msg)
         self.code = code
 
 
@@ -92,6 +95,8 @@ def load(build_if_missing: bool = True):
                                    ctypes.POINTER(i64)]
     lib.fnpu_decode_attn_noalloc.argtypes = [ctypes.POINTER(AttnDesc), i32, P, P, i32, i32, i32,
                                              P, P, P, P, P, P]
+    lib.fnpu_last_cuda_error.argtypes = []
+    lib.fnpu_last_cuda_error.restype = ctypes.c_char_p
     lib.fnpu_status_str.argtypes = [ctypes.c_int]
     lib.fnpu_status_str.restype = ctypes.c_char_p
     for name in ("fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex",
@@ -100,6 +105,10 @@ def load(build_if_missing: bool = True):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
+
+
+def last_cuda_error() -> str:
+    return load().fnpu_last_cuda_error().decode()
 
 
 def status_str(code: int) -> str:

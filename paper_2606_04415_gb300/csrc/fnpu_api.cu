@@ -8,6 +8,7 @@
 // carries metadata only; tensors stay with the caller (Sec. 3.2).
 #include <math.h>
 #include <stdlib.h>
+#include <stdio.h>
 #include <string.h>
 
 #include <algorithm>
@@ -42,6 +43,15 @@ struct fnpu_plan {
 };
 
 namespace fnpu {
+
+thread_local char g_last_cuda_error[256] = "";
+
+int cuda_fail(cudaError_t e, const char *where) {
+    snprintf(g_last_cuda_error, sizeof(g_last_cuda_error), "%s: %s", where, cudaGetErrorString(e));
+    cudaGetLastError();  // clear non-sticky errors
+    return FNPU_ECUDA;
+}
+
 namespace {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -91,6 +101,8 @@ const char *fnpu_status_str(int s) {
 }
 
 int fnpu_version(void) { return 100; }
+
+const char *fnpu_last_cuda_error(void) { return g_last_cuda_error; }
 
 int fnpu_kv_append(const fnpu_attn_desc *desc, const void *k_new, const void *v_new,
                    const int64_t *slot_mapping, int32_t num_tokens, void *k_cache, void *v_cache,
@@ -269,7 +281,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
     const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
-    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 4, 256);
+    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 4, 256);  // err + work queue
     const size_t meta_bytes = off;
     const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * G, 256);
     const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * G * desc->head_dim_v, 256);
@@ -343,6 +355,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.group = d.num_q_heads / d.num_kv_heads;
     p.block_size = d.block_size;
     p.num_blocks = d.num_blocks;
+    p.num_tokens = pl->num_tokens;
     p.head_dim_qk = d.head_dim_qk;
     p.head_dim_v = d.head_dim_v;
     p.k_slot_stride = latent ? d.head_dim_qk : static_cast<int64_t>(d.num_kv_heads) * d.head_dim_qk;
@@ -356,6 +369,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.pitems = pl->d_pitems;
     p.num_pitems = pl->num_pitems;
     p.err = pl->d_err;
+    p.sched = pl->d_err + 2;
 
     int rc = launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
@@ -369,8 +383,8 @@ int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
     int32_t v = 0;
     if (cudaMemcpy(&v, pl->d_err, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return FNPU_ECUDA;
     if (v != 0) {
-        const int32_t zero = 0;
-        if (cudaMemcpy(pl->d_err, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+        const int32_t zero[4] = {0, 0, 0, 0};  // also resets the persistent work queue
+        if (cudaMemcpy(pl->d_err, zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
             return FNPU_ECUDA;
         return FNPU_EDEVICE_TIMEOUT;
     }

@@ -1,6 +1,7 @@
 // Internal structures shared between the host planner and the kernels.
 #pragma once
 
+#include <cuda_runtime.h>
 #include <stdint.h>
 
 #include "../../include/fnpu.h"
@@ -44,6 +45,7 @@ struct AttnParams {
     const int32_t *block_table;  // [num_seqs, bt_stride]
     int32_t bt_stride;
     int32_t num_q_heads, num_kv_heads, group, block_size, num_blocks;
+    int64_t num_tokens;
     int32_t head_dim_qk, head_dim_v;
     int64_t k_slot_stride;  // elements between consecutive slots of k_cache
     int64_t v_slot_stride;
@@ -58,7 +60,16 @@ struct AttnParams {
     const PrefillItem *pitems;
     int32_t num_pitems;
     int32_t *err;           // device error flag of the plan
+    int32_t *sched;         // [2] persistent work queue: next item, finished CTAs
 };
+
+// Record a failed CUDA call for fnpu_last_cuda_error(); returns FNPU_ECUDA.
+int cuda_fail(cudaError_t e, const char *where);
+#define FNPU_CUDA_TRY(call)                                   \
+    do {                                                      \
+        cudaError_t e_ = (call);                              \
+        if (e_ != cudaSuccess) return ::fnpu::cuda_fail(e_, #call); \
+    } while (0)
 
 // Launchers (defined in the .cu files).
 int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_new,

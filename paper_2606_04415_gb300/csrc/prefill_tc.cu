@@ -4,24 +4,39 @@
 // are dense bf16 contractions, so they run as tcgen05.mma with fp32
 // accumulators in tensor memory.
 //
-// Work item: one kv head and P = floor(128 / G) consecutive query positions of
-// a prefill chunk; the 128 MMA rows are (position, query head) pairs of that
-// kv head (row = p * G + h), so every K/V byte staged in shared memory serves
-// all G heads of the group (GQA packing; 126 of 128 rows busy for G = 7).
+// GQA packing: a Q tile is 128 MMA rows = (position, query head) pairs of one
+// kv head (row = p * G + h, P = floor(128 / G) positions), so each K/V byte
+// staged in shared memory serves all G heads of the group (126 of 128 rows
+// busy for G = 7). A 3-D TMA box (64 columns x G heads x P positions) writes
+// exactly this row order. A work item is two consecutive Q tiles of one kv
+// head (2P positions) that consume the same K/V tiles, which halves the
+// L2-to-SM traffic per FLOP (one Q tile per K/V tile would need about
+// 50 B/clk per SM at the tensor rate).
 //
-// Per CTA (192 threads, two CTAs per SM):
-//   warps 0-3  one MMA row per thread: Q row into TMEM, online softmax on the
-//              S row read from TMEM, P (bf16) written back over S, lazy
-//              rescaling of the O row, epilogue;
-//   warp 4     TMA producer: 64-key K/V tiles gathered block by block through
-//              the block table (one 4-D box per block and 64-column half) into
-//              a 3-stage ring; zeroes V rows past the context in the last tile
-//              so stale slots never reach the PV product;
-//   warp 5     one thread issues the MMAs: S = Q K^T (A = Q from TMEM, B = K
-//              K-major) and O += P V (A = P from TMEM, B = V MN-major).
-// TMEM (256 columns): Q bf16 at 0, S fp32 / P bf16 at 64, O fp32 at 128.
+// One persistent CTA per SM (384 threads) takes items, longest first, from an
+// atomic queue (the last CTA to finish resets it for the next run):
+//   warps 0-3, 4-7  softmax warpgroups for Q tile 0 and tile 1, one MMA row
+//                   per thread: online softmax on the S row read from TMEM,
+//                   P (bf16) written over S, lazy rescale of the O row,
+//                   epilogue;
+//   warp 8          scheduler and K producer: the item's two Q tiles, then the
+//                   64-key K tiles gathered block by block through the block
+//                   table (one 4-D box per block and 64-column half);
+//   warp 9          V producer for the same tiles; zeroes V rows past the
+//                   context before the last PV of an item. Each TMA issue
+//                   costs on the order of a hundred cycles per issuing warp,
+//                   so K and V are issued from separate warps;
+//   warps 10, 11    issue the MMAs (warp-uniform, one elected lane); warp 10
+//                   issues S_w(j+1) = Q_w K(j+1)^T as soon as warpgroup w has
+//                   copied S_w(j) into registers, warp 11 issues
+//                   O_w += P_w(j) V(j) as soon as P_w(j) is written. The MMA
+//                   queue is short, so one warp's barrier waits would leave the
+//                   tensor core idle; two issuers keep it fed.
+// TMEM (512 columns): S0 at 0, S1 at 64 (fp32); P0 at 128/160 and P1 at
+// 192/224 (bf16, double-buffered); O0 at 256, O1 at 384. Because P has its
+// own buffers, no S MMA ever waits for a PV to drain.
 // Every mbarrier wait is bounded; a timeout raises the plan's error flag and
-// the CTA drains, frees its tensor memory and exits.
+// the CTA drains its tensor-core work, frees its tensor memory and exits.
 #include <math.h>
 
 #include <mutex>
@@ -32,67 +47,113 @@
 namespace fnpu {
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 384;
 constexpr int kRows = 128;
 constexpr int kKeys = 64;
-constexpr int kStages = 3;
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColQ = 0, kColS = 64, kColO = 128;
+constexpr int kStages = 4;
+constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p <= 2^8 before a rescale
+
+__host__ __device__ constexpr uint32_t col_s(int w) { return 64u * w; }
+__host__ __device__ constexpr uint32_t col_p(int w, int b) { return 128u + 64u * w + 32u * b; }
+__host__ __device__ constexpr uint32_t col_o(int w) { return 256u + 128u * w; }
 
 template <int D>
 struct TcCfg {
     static constexpr int kTileBytes = kKeys * D * 2;  // one K or V tile
     static constexpr int kStageBytes = 2 * kTileBytes;
-    static constexpr int kHalf = kKeys * 128;         // one 64-column half of a tile
-    // barriers: kfull[3], vfull[3], kvempty[3], sfull, pfull, pvdone, qready, vzero, drain
-    static constexpr int kNumBars = 3 * kStages + 6;
-    static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + 8 * kNumBars + 16;
+    static constexpr int kHalf = kKeys * 128;         // one 64-column half of a K/V tile
+    static constexpr int kQHalf = kRows * 128;        // one 64-column half of a Q tile
+    static constexpr int kQBytes = kRows * D * 2;     // one Q tile
+    static constexpr int kQOff = kStages * kStageBytes;
+    static constexpr int kBarOff = kQOff + 2 * kQBytes;
+    // kfull[S] vfull[S] kempty[S] vempty[S] sfull[2] sfree[2] pfull[2][2] pvdone[2][2]
+    // qfull qempty vzero itemfull[2] itemempty[2] drain[2]
+    static constexpr int kNumBars = 4 * kStages + 12 + 9;
+    static constexpr int kSmemUsed = 1024 + kBarOff + 8 * kNumBars + 32;
+    // at least 116 KB so that no two CTAs share an SM (each holds all 512 TMEM columns)
+    static constexpr int kSmemBytes = kSmemUsed > 116 * 1024 ? kSmemUsed : 116 * 1024;
+    static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 };
 
 struct TcMaps {
-    CUtensorMap k, v;
+    CUtensorMap k, v, q;
 };
 
+struct ItemGeom {
+    int kvh, p0, rows, prefix, ctx, ntiles, q_start, bt_row;
+    bool tail_fix;
+};
+
+__device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
+    const PrefillItem it = p.pitems[idx];
+    const SeqInfo si = p.seqs[it.seq];
+    ItemGeom g;
+    g.kvh = it.head;
+    g.p0 = it.row_begin;
+    g.rows = it.rows;
+    g.prefix = si.ctx_len - si.q_len;
+    g.ctx = si.ctx_len;
+    const int nkeys = g.prefix + it.row_begin + it.rows;  // keys 0 .. last position
+    g.ntiles = (nkeys + kKeys - 1) / kKeys;
+    g.q_start = si.q_start;
+    g.bt_row = si.bt_row;
+    g.tail_fix = g.ntiles * kKeys > g.ctx;
+    return g;
+}
+
 template <int D>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
     prefill_tc_kernel(const AttnParams p, const __grid_constant__ TcMaps maps) {
     using Cfg = TcCfg<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t s_base = smem_u32(smem);
-    const uint32_t s_bars = s_base + kStages * Cfg::kStageBytes;
+    const uint32_t s_bars = s_base + Cfg::kBarOff;
     auto KFULL = [&](int s) { return s_bars + 8 * s; };
     auto VFULL = [&](int s) { return s_bars + 8 * (kStages + s); };
-    auto KVEMPTY = [&](int s) { return s_bars + 8 * (2 * kStages + s); };
-    const uint32_t SFULL = s_bars + 8 * (3 * kStages), PFULL = SFULL + 8, PVDONE = SFULL + 16,
-                   QREADY = SFULL + 24, VZERO = SFULL + 32, DRAIN = SFULL + 40;
-    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(smem + kStages * Cfg::kStageBytes + 8 * Cfg::kNumBars);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kStages * Cfg::kStageBytes + 8 * Cfg::kNumBars + 4);
+    auto KEMPTY = [&](int s) { return s_bars + 8 * (2 * kStages + s); };
+    auto VEMPTY = [&](int s) { return s_bars + 8 * (3 * kStages + s); };
+    const uint32_t b0 = s_bars + 8 * (4 * kStages);
+    auto SFULL = [&](int w) { return b0 + 8 * w; };
+    auto SFREE = [&](int w) { return b0 + 16 + 8 * w; };
+    auto PFULL = [&](int w, int b) { return b0 + 32 + 8 * (2 * w + b); };
+    auto PVDONE = [&](int w, int b) { return b0 + 64 + 8 * (2 * w + b); };
+    const uint32_t QFULL = b0 + 96, QEMPTY = b0 + 104, VZERO = b0 + 112;
+    auto ITEMFULL = [&](int k) { return b0 + 120 + 8 * k; };
+    auto ITEMEMPTY = [&](int k) { return b0 + 136 + 8 * k; };
+    auto DRAIN = [&](int i) { return b0 + 152 + 8 * i; };
+    uint8_t *misc = smem + Cfg::kBarOff + 8 * Cfg::kNumBars;
+    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(misc);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 4);
+    volatile int *item_slot = reinterpret_cast<volatile int *>(misc + 8);  // [2]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const PrefillItem it = p.pitems[blockIdx.x];
-    const SeqInfo si = p.seqs[it.seq];
     const int G = p.group;
-    const int kvh = it.head;
-    const int prefix = si.ctx_len - si.q_len;
-    const int nkeys = prefix + it.row_begin + it.rows;  // keys 0 .. last position
-    const int ntiles = (nkeys + kKeys - 1) / kKeys;
-    const int ctx = si.ctx_len;
-    const bool tail_fix = ntiles * kKeys > ctx;
+    const int P = kRows / G;
 
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(KFULL(s), 1);
             tc::mbar_init(VFULL(s), 1);
-            tc::mbar_init(KVEMPTY(s), 1);
+            tc::mbar_init(KEMPTY(s), 1);
+            tc::mbar_init(VEMPTY(s), 1);
         }
-        tc::mbar_init(SFULL, 1);
-        tc::mbar_init(PFULL, kRows);
-        tc::mbar_init(PVDONE, 1);
-        tc::mbar_init(QREADY, kRows);
+        for (int w = 0; w < 2; ++w) {
+            tc::mbar_init(SFULL(w), 1);
+            tc::mbar_init(SFREE(w), kRows);
+            for (int b = 0; b < 2; ++b) {
+                tc::mbar_init(PFULL(w, b), kRows);
+                tc::mbar_init(PVDONE(w, b), 1);
+            }
+            tc::mbar_init(ITEMFULL(w), 1);
+            tc::mbar_init(ITEMEMPTY(w), 3 + 2 * kRows);  // two MMA issuers, V producer, 256 softmax rows
+        }
+        tc::mbar_init(QFULL, 1);
+        tc::mbar_init(QEMPTY, 1);
         tc::mbar_init(VZERO, 1);
-        tc::mbar_init(DRAIN, 1);
+        tc::mbar_init(DRAIN(0), 1);
+        tc::mbar_init(DRAIN(1), 1);
         *abort_flag = 0;
         tc::fence_mbar_init();
     }
@@ -105,6 +166,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const uint32_t tmem = *tmem_slot;
 
     auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
+        if (tc::mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
         if (tc::mbar_wait(bar, parity)) return true;
         *abort_flag = 1;
@@ -112,205 +174,291 @@ __global__ void __launch_bounds__(kThreads, 2)
         return false;
     };
 
-    if (warp == 4) {
-        // ------------------------------------------------------------ producer
-        const int32_t *bt = p.block_table + static_cast<int64_t>(si.bt_row) * p.bt_stride;
+    if (warp == 8 || warp == 9) {
+        // ---------------------------------- producers (8: scheduler, Q, K; 9: V)
+        const bool is_k = warp == 8;
+        if (lane == 0) {
+            tc::prefetch_tmap(is_k ? &maps.k : &maps.v);
+            if (is_k) tc::prefetch_tmap(&maps.q);
+        }
         const int bs = p.block_size;
-        const int nblk_seq = (ctx + bs - 1) / bs;
         const int per_tile = kKeys / bs;
-        if (lane == 0) {
-            tc::prefetch_tmap(&maps.k);
-            tc::prefetch_tmap(&maps.v);
-        }
-        for (int i = 0; i < ntiles; ++i) {
-            const int st = i % kStages;
-            if (i >= kStages && !wait(KVEMPTY(st), ((i / kStages) - 1) & 1)) break;
-            const int jb = i * per_tile;
-            int nvalid = nblk_seq - jb;
-            nvalid = nvalid < 0 ? 0 : (nvalid > per_tile ? per_tile : nvalid);
-            const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
-            if (lane == 0) {
-                const uint32_t bytes = static_cast<uint32_t>(nvalid) * bs * D * 2;
-                tc::mbar_arrive_expect_tx(KFULL(st), bytes);
-                for (int b = 0; b < nvalid; ++b) {
-                    const int blk = __ldg(bt + jb + b);
-#pragma unroll
-                    for (int h = 0; h < D / 64; ++h)
-                        tc::tma_load_4d(sK + h * Cfg::kHalf + b * bs * 128, &maps.k, KFULL(st), h * 64, kvh, 0, blk);
+        const CUtensorMap *map = is_k ? &maps.k : &maps.v;
+        int g = 0;  // tiles issued so far (stage ring position)
+        int nfix = 0;
+        for (int k = 0;; ++k) {
+            const int slot = k & 1;
+            int idx = 0;
+            if (is_k) {
+                if (lane == 0) idx = atomicAdd(p.sched, 1);
+                idx = __shfl_sync(0xffffffffu, idx, 0);
+                if (k >= 2 && !wait(ITEMEMPTY(slot), ((k >> 1) - 1) & 1)) break;
+                if (lane == 0) {
+                    item_slot[slot] = idx < p.num_pitems ? idx : -1;
+                    tc::mbar_arrive(ITEMFULL(slot));
                 }
-                tc::mbar_arrive_expect_tx(VFULL(st), bytes);
-                for (int b = 0; b < nvalid; ++b) {
-                    const int blk = __ldg(bt + jb + b);
-#pragma unroll
-                    for (int h = 0; h < D / 64; ++h)
-                        tc::tma_load_4d(sV + h * Cfg::kHalf + b * bs * 128, &maps.v, VFULL(st), h * 64, kvh, 0, blk);
-                }
-            }
-            __syncwarp();
-            if (i == ntiles - 1 && tail_fix) {
-                // zero V rows of keys >= ctx (stale slots, unloaded blocks)
-                if (!wait(VFULL(st), (i / kStages) & 1)) break;
-                const int r0 = ctx - i * kKeys;
-                const int nrows = kKeys - r0;
-                for (int idx = lane; idx < nrows * 8 * (D / 64); idx += 32) {
-                    const int h = idx / (nrows * 8), rem = idx % (nrows * 8);
-                    const int row = r0 + rem / 8, ch = rem % 8;
-                    *reinterpret_cast<uint4 *>(smem + st * Cfg::kStageBytes + Cfg::kTileBytes + h * Cfg::kHalf +
-                                               row * 128 + ch * 16) = make_uint4(0u, 0u, 0u, 0u);
-                }
-                tc::fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) tc::mbar_arrive(VZERO);
-            }
-        }
-    } else if (warp == 5) {
-        // ---------------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idS = tc::idesc_bf16(kRows, kKeys, false);
-            constexpr uint32_t idO = tc::idesc_bf16(kRows, D, true);
-            bool ok = wait(QREADY, 0);
-            int issued = 0;
-            for (int i = 0; ok && i < ntiles; ++i) {
-                const int st = i % kStages;
-                const uint32_t ph = (i / kStages) & 1;
-                if (!wait(KFULL(st), ph)) { ok = false; break; }
-                if (i > 0 && !wait(PVDONE, (i - 1) & 1)) { ok = false; break; }
-                tc::fence_after_sync();
-                const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint64_t b = tc::sdesc_sw128(sK + (kk / 4) * Cfg::kHalf + (kk % 4) * 32, 16, 1024);
-                    tc::mma_ts(tmem + kColS, tmem + kColQ + kk * 8, b, idS, kk > 0);
-                }
-                tc::commit(SFULL);
-                issued = 1;
-                if (!wait(PFULL, i & 1)) { ok = false; break; }
-                if (i == ntiles - 1 && tail_fix) {
-                    if (!wait(VZERO, 0)) { ok = false; break; }
-                } else if (!wait(VFULL(st), ph)) {
-                    ok = false;
-                    break;
-                }
-                tc::fence_after_sync();
-#pragma unroll
-                for (int kk = 0; kk < kKeys / 16; ++kk) {
-                    const uint64_t b = tc::sdesc_sw128(sV + kk * 2048, Cfg::kHalf, 1024);
-                    tc::mma_ts(tmem + kColO, tmem + kColS + kk * 8, b, idO, (i > 0 || kk > 0) ? 1u : 0u);
-                }
-                tc::commit(KVEMPTY(st));
-                tc::commit(PVDONE);
-            }
-            if (!ok && issued) {  // drain whatever is still in flight
-                tc::commit(DRAIN);
-                tc::mbar_wait(DRAIN, 0, 200000000ull);
-            }
-        }
-        __syncwarp();
-    } else {
-        // ------------------------------------------- softmax / epilogue rows
-        const int r = tid;  // MMA row = TMEM lane
-        const int P = kRows / G;
-        const int pl = r / G, hl = r % G;
-        const bool row_ok = (r < P * G) && (pl < it.rows);
-        // rows past the item (padding) keep a position too; their results are
-        // never stored, so they need no masking of their own
-        const int pos = prefix + it.row_begin + pl;
-        const int min_pos = prefix + it.row_begin;
-        const int64_t tok = si.q_start + it.row_begin + pl;
-        const int head = kvh * G + hl;
-        const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-
-        {  // Q row -> TMEM (bf16 pairs), zeros for padding rows
-            const uint4 *q = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(p.q) +
-                                                             (tok * p.num_q_heads + head) * D);
-#pragma unroll
-            for (int c = 0; c < D / 64; ++c) {
-                uint32_t v[32];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    uint4 x = row_ok ? __ldg(q + c * 8 + j) : make_uint4(0u, 0u, 0u, 0u);
-                    v[4 * j] = x.x; v[4 * j + 1] = x.y; v[4 * j + 2] = x.z; v[4 * j + 3] = x.w;
-                }
-                tc::tmem_st32(lane_addr + kColQ + 32 * c, v);
-            }
-            tc::tmem_wait_st();
-            tc::fence_before_sync();
-            tc::mbar_arrive(QREADY);
-        }
-
-        float m_run = -INFINITY;  // reference max (log2 units) of the exponentials
-        float l = 0.f;
-        bool ok = true;
-        for (int i = 0; i < ntiles; ++i) {
-            if (!wait(SFULL, i & 1)) { ok = false; break; }
-            tc::fence_after_sync();
-            uint32_t s[64];
-            tc::tmem_ld32(lane_addr + kColS, *reinterpret_cast<uint32_t(*)[32]>(&s[0]));
-            tc::tmem_ld32(lane_addr + kColS + 32, *reinterpret_cast<uint32_t(*)[32]>(&s[32]));
-            tc::tmem_wait_ld();
-            // tiles that reach past the first row's position need the causal
-            // mask; all others are fully visible to every row of the item
-            const int k0 = i * kKeys;
-            const bool masked_tile = k0 + kKeys - 1 > min_pos;
-            float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
-            if (masked_tile) {
-#pragma unroll
-                for (int j = 0; j < kKeys; j += 4) {
-                    float v0 = __uint_as_float(s[j]), v1 = __uint_as_float(s[j + 1]);
-                    float v2 = __uint_as_float(s[j + 2]), v3 = __uint_as_float(s[j + 3]);
-                    v0 = (k0 + j <= pos) ? v0 : -INFINITY;
-                    v1 = (k0 + j + 1 <= pos) ? v1 : -INFINITY;
-                    v2 = (k0 + j + 2 <= pos) ? v2 : -INFINITY;
-                    v3 = (k0 + j + 3 <= pos) ? v3 : -INFINITY;
-                    s[j] = __float_as_uint(v0); s[j + 1] = __float_as_uint(v1);
-                    s[j + 2] = __float_as_uint(v2); s[j + 3] = __float_as_uint(v3);
-                    mx0 = fmaxf(mx0, v0); mx1 = fmaxf(mx1, v1); mx2 = fmaxf(mx2, v2); mx3 = fmaxf(mx3, v3);
-                }
+                if (idx >= p.num_pitems) break;
             } else {
-#pragma unroll
-                for (int j = 0; j < kKeys; j += 4) {
-                    mx0 = fmaxf(mx0, __uint_as_float(s[j])); mx1 = fmaxf(mx1, __uint_as_float(s[j + 1]));
-                    mx2 = fmaxf(mx2, __uint_as_float(s[j + 2])); mx3 = fmaxf(mx3, __uint_as_float(s[j + 3]));
-                }
+                if (!wait(ITEMFULL(slot), (k >> 1) & 1)) break;
+                idx = __shfl_sync(0xffffffffu, item_slot[slot], 0);
+                if (idx < 0) break;
             }
-            // the scale is positive, so the max of scaled scores is the scaled max
-            const float tmax = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * p.scale_log2;
-            const bool need = (m_run == -INFINITY) ? (tmax != -INFINITY) : (tmax > m_run + kRescaleThreshold);
-            if (__any_sync(0xffffffffu, need)) {
-                const float m_new = need ? fmaxf(m_run, tmax) : m_run;
-                const float alpha = (need && m_run != -INFINITY) ? fast_exp2(m_run - m_new) : 1.f;
-                if (i > 0) {  // O of the previous tiles is complete (S(i) was issued after PV(i-1))
+            const ItemGeom it = item_geom(p, idx);
+            const int ukvh = __shfl_sync(0xffffffffu, it.kvh, 0);
+            if (is_k) {  // both Q tiles, once the previous item's last S is done
+                if (k >= 1 && !wait(QEMPTY, (k - 1) & 1)) break;
+                tc::mbar_arrive_expect_tx_warp(QFULL, static_cast<uint32_t>(2 * (D / 64) * 64 * G * P * 2));
+                const int q0 = __shfl_sync(0xffffffffu, it.q_start + it.p0, 0);
 #pragma unroll
-                    for (int c = 0; c < D / 32; ++c) {
-                        uint32_t o[32];
-                        tc::tmem_ld32(lane_addr + kColO + 32 * c, o);
-                        tc::tmem_wait_ld();
+                for (int w = 0; w < 2; ++w)
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
-                        tc::tmem_st32(lane_addr + kColO + 32 * c, o);
+                    for (int h = 0; h < D / 64; ++h)
+                        tc::tma_load_3d_warp(s_base + Cfg::kQOff + w * Cfg::kQBytes + h * Cfg::kQHalf, &maps.q,
+                                             QFULL, h * 64, ukvh * G, q0 + w * P);
+            }
+            const int32_t *bt = p.block_table + static_cast<int64_t>(it.bt_row) * p.bt_stride;
+            const int nblk_seq = (it.ctx + bs - 1) / bs;
+            // block ids of the next tile, one per lane, loaded a tile ahead so
+            // that the TMA issue never waits on a block-table read
+            int blk_next = (lane < per_tile && lane < nblk_seq) ? __ldg(bt + lane) : 0;
+            bool ok = true;
+            for (int i = 0; i < it.ntiles; ++i, ++g) {
+                const int st = g % kStages;
+                const int blk_cur = blk_next;
+                const int jn = (i + 1) * per_tile + lane;
+                blk_next = (i + 1 < it.ntiles && lane < per_tile && jn < nblk_seq) ? __ldg(bt + jn) : 0;
+                if (g >= kStages && !wait(is_k ? KEMPTY(st) : VEMPTY(st), ((g / kStages) - 1) & 1)) { ok = false; break; }
+                int nvalid = nblk_seq - i * per_tile;
+                nvalid = nvalid < 0 ? 0 : (nvalid > per_tile ? per_tile : nvalid);
+                nvalid = __shfl_sync(0xffffffffu, nvalid, 0);
+                const uint32_t dst = s_base + st * Cfg::kStageBytes + (is_k ? 0 : Cfg::kTileBytes);
+                const uint32_t bar = is_k ? KFULL(st) : VFULL(st);
+                tc::mbar_arrive_expect_tx_warp(bar, static_cast<uint32_t>(nvalid) * bs * D * 2);
+#pragma unroll
+                for (int b = 0; b < 4; ++b) {
+                    const int blk = __shfl_sync(0xffffffffu, blk_cur, b);
+                    if (b < nvalid) {
+#pragma unroll
+                        for (int h = 0; h < D / 64; ++h)
+                            tc::tma_load_4d_warp(dst + h * Cfg::kHalf + b * bs * 128, map, bar, h * 64, ukvh, 0, blk);
                     }
                 }
-                l *= alpha;
-                m_run = m_new;
+                if (!is_k && i == it.ntiles - 1 && it.tail_fix) {
+                    // zero V rows of keys >= ctx (stale slots, unloaded blocks)
+                    if (!wait(VFULL(st), (g / kStages) & 1)) { ok = false; break; }
+                    const int r0 = it.ctx - i * kKeys;
+                    const int nrows = kKeys - r0;
+                    for (int e = lane; e < nrows * 8 * (D / 64); e += 32) {
+                        const int h = e / (nrows * 8), rem = e % (nrows * 8);
+                        const int row = r0 + rem / 8, ch = rem % 8;
+                        *reinterpret_cast<uint4 *>(smem + st * Cfg::kStageBytes + Cfg::kTileBytes + h * Cfg::kHalf +
+                                                   row * 128 + ch * 16) = make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    tc::fence_proxy_async_smem();
+                    __syncwarp();
+                    tc::mbar_arrive_warp(VZERO);
+                    ++nfix;
+                }
             }
-            const float nbase = (m_run == -INFINITY) ? 0.f : -m_run;
-            const float sc = p.scale_log2;
-            float l0 = 0.f, l1 = 0.f;
-            uint32_t pk[32];
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * j]), sc, nbase));
-                const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * j + 1]), sc, nbase));
-                if (j & 1) l1 += p0 + p1; else l0 += p0 + p1;
-                pk[j] = pack_bf16x2(p0, p1);
-            }
-            l += l0 + l1;
-            tc::tmem_st32(lane_addr + kColS, pk);
-            tc::tmem_wait_st();
-            tc::fence_before_sync();
-            tc::mbar_arrive(PFULL);
+            if (!ok) break;
+            if (!is_k) tc::mbar_arrive_warp(ITEMEMPTY(slot));
         }
-        if (ok && wait(PVDONE, (ntiles - 1) & 1)) {
+    } else if (warp == 10 || warp == 11) {
+        // ------------------------------------------------------- MMA issuers
+        // Each warp runs its loop with warp-uniform values (passed through
+        // __shfl_sync so the compiler keeps them in uniform registers); each
+        // tcgen05 instruction is issued by one elected lane. Warp 10 issues the
+        // S products, warp 11 the PV products; tcgen05.commit tracks only the
+        // issuing warp's own MMAs, so each warp commits its own barriers.
+        const bool s_issuer = warp == 10;
+        constexpr uint32_t idS = tc::idesc_bf16(kRows, kKeys, false);
+        constexpr uint32_t idO = tc::idesc_bf16(kRows, D, true);
+        const uint32_t utmem = __shfl_sync(0xffffffffu, tmem, 0);
+        const uint32_t us_base = __shfl_sync(0xffffffffu, s_base, 0);
+        int g = 0, t = 0, nfix = 0;
+        bool ok = true, issued = false;
+        auto issue_s = [&](int w, int st_in) {
+            const int st = __shfl_sync(0xffffffffu, st_in, 0);
+            const uint64_t kd = tc::sdesc_sw128(us_base + st * Cfg::kStageBytes, 16, 1024);
+            const uint64_t qd = tc::sdesc_sw128(us_base + Cfg::kQOff + w * Cfg::kQBytes, 16, 1024);
+            const uint32_t dS = utmem + col_s(w);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                tc::mma_ss_warp(dS, qd + ((kk / 4) * Cfg::kQHalf + (kk % 4) * 32) / 16,
+                                kd + ((kk / 4) * Cfg::kHalf + (kk % 4) * 32) / 16, idS, kk > 0);
+            tc::commit_warp(SFULL(w));
+        };
+        auto issue_pv = [&](int w, int st_in, int b_in, uint32_t acc_in) {
+            const int st = __shfl_sync(0xffffffffu, st_in, 0);
+            const int b = __shfl_sync(0xffffffffu, b_in, 0);
+            const uint32_t acc = __shfl_sync(0xffffffffu, acc_in, 0);
+            const uint64_t vd = tc::sdesc_sw128(us_base + st * Cfg::kStageBytes + Cfg::kTileBytes, Cfg::kHalf, 1024);
+            const uint32_t dO = utmem + col_o(w), aP = utmem + col_p(w, 0) + 32u * b;
+            tc::mma_ts_warp(dO, aP, vd, idO, acc);
+#pragma unroll
+            for (int kk = 1; kk < kKeys / 16; ++kk) tc::mma_ts_warp(dO, aP + kk * 8, vd + (kk * 2048) / 16, idO, 1u);
+            tc::commit_warp(PVDONE(w, b));
+        };
+        for (int k = 0; ok; ++k) {
+            const int slot = k & 1;
+            if (!wait(ITEMFULL(slot), (k >> 1) & 1)) { ok = false; break; }
+            const int idx = __shfl_sync(0xffffffffu, item_slot[slot], 0);
+            if (idx < 0) break;
+            const ItemGeom it = item_geom(p, idx);
+            const int n = __shfl_sync(0xffffffffu, it.ntiles, 0);
+            const bool tail = __shfl_sync(0xffffffffu, it.tail_fix ? 1 : 0, 0) != 0;
+            if (s_issuer) {
+                if (!wait(QFULL, k & 1)) { ok = false; break; }
+                for (int j = 0; j < n; ++j) {
+                    const int T = t + j, gj = g + j, st = gj % kStages;
+                    if (!wait(KFULL(st), (gj / kStages) & 1)) { ok = false; break; }
+                    // S_w(T) overwrites S_w(T - 1), which warpgroup w has copied out
+                    if (T >= 1 && !wait(SFREE(0), (T - 1) & 1)) { ok = false; break; }
+                    tc::fence_after_sync();
+                    issue_s(0, st);
+                    issued = true;
+                    if (T >= 1 && !wait(SFREE(1), (T - 1) & 1)) { ok = false; break; }
+                    tc::fence_after_sync();
+                    issue_s(1, st);
+                    tc::commit_warp(KEMPTY(st));
+                    if (j == n - 1) tc::commit_warp(QEMPTY);  // last S of this item
+                }
+            } else {
+                for (int j = 0; j < n; ++j) {
+                    const int T = t + j, gj = g + j, st = gj % kStages;
+                    if (j == n - 1 && tail) {
+                        if (!wait(VZERO, nfix & 1)) { ok = false; break; }
+                    } else if (!wait(VFULL(st), (gj / kStages) & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    if (!wait(PFULL(0, T & 1), (T >> 1) & 1)) { ok = false; break; }
+                    tc::fence_after_sync();
+                    issue_pv(0, st, T & 1, j > 0 ? 1u : 0u);
+                    issued = true;
+                    if (!wait(PFULL(1, T & 1), (T >> 1) & 1)) { ok = false; break; }
+                    tc::fence_after_sync();
+                    issue_pv(1, st, T & 1, j > 0 ? 1u : 0u);
+                    tc::commit_warp(VEMPTY(st));
+                }
+            }
+            if (!ok) break;
+            g += n;
+            t += n;
+            if (tail) ++nfix;
+            tc::mbar_arrive_warp(ITEMEMPTY(slot));
+        }
+        if (!ok && issued) {  // drain whatever this warp still has in flight
+            tc::commit_warp(DRAIN(s_issuer ? 0 : 1));
+            tc::mbar_wait(DRAIN(s_issuer ? 0 : 1), 0, 200000000ull);
+        }
+    } else {
+        // ------------------------------------------- softmax / epilogue rows
+        const int w = warp >> 2;                 // warpgroup = Q tile
+        const int r = tid & 127;                 // MMA row = TMEM lane
+        const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+        const int pl = r / G, hl = r % G;
+        const float sc = p.scale_log2;
+        int t = 0;
+        for (int k = 0;; ++k) {
+            const int slot = k & 1;
+            if (!wait(ITEMFULL(slot), (k >> 1) & 1)) break;
+            const int idx = item_slot[slot];
+            if (idx < 0) break;
+            const ItemGeom it = item_geom(p, idx);
+            const int pw = it.p0 + w * P;
+            const bool row_ok = (r < P * G) && (pw + pl < it.p0 + it.rows);
+            // rows past the item (padding) keep a position too; their results are
+            // never stored, so they need no masking of their own
+            const int pos = it.prefix + pw + pl;
+            const int min_pos = it.prefix + pw;
+            const int64_t tok = it.q_start + pw + pl;
+            const int head = it.kvh * G + hl;
+
+            float m_run = -INFINITY;  // reference max (log2 units) of the exponentials
+            float l = 0.f;
+            bool ok = true;
+            for (int i = 0; i < it.ntiles; ++i) {
+                const int T = t + i, b = T & 1;
+                if (!wait(SFULL(w), T & 1)) { ok = false; break; }
+                tc::fence_after_sync();
+                uint32_t s[64];
+                tc::tmem_ld32(lane_addr + col_s(w), *reinterpret_cast<uint32_t(*)[32]>(&s[0]));
+                tc::tmem_ld32(lane_addr + col_s(w) + 32, *reinterpret_cast<uint32_t(*)[32]>(&s[32]));
+                tc::tmem_wait_ld();
+                tc::fence_before_sync();
+                tc::mbar_arrive(SFREE(w));  // the S buffer may be overwritten now
+                // tiles that reach past the first row's position need the causal
+                // mask; all others are fully visible to every row of the tile
+                const int k0 = i * kKeys;
+                const bool masked_tile = k0 + kKeys - 1 > min_pos;
+                float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+                if (masked_tile) {
+#pragma unroll
+                    for (int j = 0; j < kKeys; j += 4) {
+                        float v0 = __uint_as_float(s[j]), v1 = __uint_as_float(s[j + 1]);
+                        float v2 = __uint_as_float(s[j + 2]), v3 = __uint_as_float(s[j + 3]);
+                        v0 = (k0 + j <= pos) ? v0 : -INFINITY;
+                        v1 = (k0 + j + 1 <= pos) ? v1 : -INFINITY;
+                        v2 = (k0 + j + 2 <= pos) ? v2 : -INFINITY;
+                        v3 = (k0 + j + 3 <= pos) ? v3 : -INFINITY;
+                        s[j] = __float_as_uint(v0); s[j + 1] = __float_as_uint(v1);
+                        s[j + 2] = __float_as_uint(v2); s[j + 3] = __float_as_uint(v3);
+                        mx0 = fmaxf(mx0, v0); mx1 = fmaxf(mx1, v1); mx2 = fmaxf(mx2, v2); mx3 = fmaxf(mx3, v3);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < kKeys; j += 4) {
+                        mx0 = fmaxf(mx0, __uint_as_float(s[j])); mx1 = fmaxf(mx1, __uint_as_float(s[j + 1]));
+                        mx2 = fmaxf(mx2, __uint_as_float(s[j + 2])); mx3 = fmaxf(mx3, __uint_as_float(s[j + 3]));
+                    }
+                }
+                // the scale is positive, so the max of scaled scores is the scaled max
+                const float tmax = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sc;
+                const bool need = (m_run == -INFINITY) ? (tmax != -INFINITY) : (tmax > m_run + kRescaleThreshold);
+                if (__any_sync(0xffffffffu, need)) {
+                    const float m_new = need ? fmaxf(m_run, tmax) : m_run;
+                    const float alpha = (need && m_run != -INFINITY) ? fast_exp2(m_run - m_new) : 1.f;
+                    if (i > 0) {  // rescale O_w once PV_w of the previous tile has landed
+                        if (!wait(PVDONE(w, (T - 1) & 1), ((T - 1) >> 1) & 1)) { ok = false; break; }
+                        tc::fence_after_sync();
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            uint32_t o[32];
+                            tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
+                            tc::tmem_wait_ld();
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
+                            tc::tmem_st32(lane_addr + col_o(w) + 32 * c, o);
+                        }
+                    }
+                    l *= alpha;
+                    m_run = m_new;
+                }
+                const float nbase = (m_run == -INFINITY) ? 0.f : -m_run;
+                // P buffer b last held P(T - 2): wait until PV(T - 2) has read it
+                if (T >= 2 && !wait(PVDONE(w, b), ((T - 2) >> 1) & 1)) { ok = false; break; }
+                float l0 = 0.f, l1 = 0.f;
+#pragma unroll
+                for (int hlf = 0; hlf < 2; ++hlf) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const float p0 = fast_exp2(fmaf(__uint_as_float(s[32 * hlf + 2 * j]), sc, nbase));
+                        const float p1 = fast_exp2(fmaf(__uint_as_float(s[32 * hlf + 2 * j + 1]), sc, nbase));
+                        if (j & 1) l1 += p0 + p1; else l0 += p0 + p1;
+                        pk[j] = pack_bf16x2(p0, p1);
+                    }
+                    tc::tmem_st16(lane_addr + col_p(w, b) + 16 * hlf, pk);
+                }
+                l += l0 + l1;
+                tc::tmem_wait_st();
+                tc::fence_before_sync();
+                tc::mbar_arrive(PFULL(w, b));
+            }
+            if (!ok) break;
+            const int Tl = t + it.ntiles - 1;
+            if (!wait(PVDONE(w, Tl & 1), (Tl >> 1) & 1)) break;
             tc::fence_after_sync();
             const float inv = 1.f / l;
             uint4 *orow = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
@@ -318,21 +466,24 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t o[32];
-                tc::tmem_ld32(lane_addr + kColO + 32 * c, o);
+                tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
                 tc::tmem_wait_ld();
                 if (row_ok) {
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        uint4 w;
-                        w.x = pack_bf16x2(__uint_as_float(o[8 * j + 0]) * inv, __uint_as_float(o[8 * j + 1]) * inv);
-                        w.y = pack_bf16x2(__uint_as_float(o[8 * j + 2]) * inv, __uint_as_float(o[8 * j + 3]) * inv);
-                        w.z = pack_bf16x2(__uint_as_float(o[8 * j + 4]) * inv, __uint_as_float(o[8 * j + 5]) * inv);
-                        w.w = pack_bf16x2(__uint_as_float(o[8 * j + 6]) * inv, __uint_as_float(o[8 * j + 7]) * inv);
-                        orow[c * 4 + j] = w;
+                        uint4 v;
+                        v.x = pack_bf16x2(__uint_as_float(o[8 * j + 0]) * inv, __uint_as_float(o[8 * j + 1]) * inv);
+                        v.y = pack_bf16x2(__uint_as_float(o[8 * j + 2]) * inv, __uint_as_float(o[8 * j + 3]) * inv);
+                        v.z = pack_bf16x2(__uint_as_float(o[8 * j + 4]) * inv, __uint_as_float(o[8 * j + 5]) * inv);
+                        v.w = pack_bf16x2(__uint_as_float(o[8 * j + 6]) * inv, __uint_as_float(o[8 * j + 7]) * inv);
+                        orow[c * 4 + j] = v;
                     }
                 }
             }
             if (row_ok) p.lse[tok * p.num_q_heads + head] = (m_run + log2f(l)) * kLn2;
+            t += it.ntiles;
+            tc::fence_before_sync();
+            tc::mbar_arrive(ITEMEMPTY(slot));
         }
     }
 
@@ -341,6 +492,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (warp == 0) {
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, kTmemCols);
+    }
+    if (tid == 0) {  // the last CTA out resets the work queue for the next run
+        __threadfence();
+        if (atomicAdd(p.sched + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+            p.sched[0] = 0;
+            p.sched[1] = 0;
+            __threadfence();
+        }
     }
 }
 
@@ -379,18 +538,37 @@ bool encode_cache_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, 
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D map over q [T, Hq, d]: box = 64 columns x G heads x P positions, so a
+// box lands as the packed (position, head) rows of one Q tile.
+bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, int G, int P) {
+    EncodeTiledFn enc = get_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(hq), static_cast<cuuint64_t>(T)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(hq) * d * 2};
+    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(P)};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int D>
 int launch_tc(const AttnParams &p, cudaStream_t st) {
     using Cfg = TcCfg<D>;
     TcMaps maps;
     if (!encode_cache_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
-        !encode_cache_map(&maps.v, p.v_cache, D, p.num_kv_heads, p.block_size, p.num_blocks))
-        return FNPU_ECUDA;
-    if (cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes) !=
-        cudaSuccess)
-        return FNPU_ECUDA;
-    prefill_tc_kernel<D><<<p.num_pitems, kThreads, Cfg::kSmemBytes, st>>>(p, maps);
-    return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
+        !encode_cache_map(&maps.v, p.v_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
+        !encode_q_map(&maps.q, p.q, D, p.num_q_heads, p.num_tokens, p.group, kRows / p.group))
+        return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Cfg::kSmemBytes));
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = p.num_pitems < sms ? p.num_pitems : sms;
+    prefill_tc_kernel<D><<<grid, kThreads, Cfg::kSmemBytes, st>>>(p, maps);
+    FNPU_CUDA_TRY(cudaGetLastError());
+    return FNPU_OK;
 }
 
 }  // namespace
@@ -400,7 +578,8 @@ bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group) {
            (block_size == 16 || block_size == 32 || block_size == 64) && group >= 1 && group <= kRows;
 }
 
-int prefill_tc_rows_per_item(int group) { return kRows / group; }
+// positions per work item: two Q tiles of floor(128 / G) positions each
+int prefill_tc_rows_per_item(int group) { return 2 * (kRows / group); }
 
 int launch_prefill_tc(const AttnParams &p, void *stream) {
     if (p.num_pitems == 0) return FNPU_OK;
