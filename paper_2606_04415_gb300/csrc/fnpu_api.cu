@@ -28,6 +28,7 @@ struct fnpu_plan {
     int32_t num_sms = 0;
     int32_t flags = 0;
     bool use_tc = false;
+    bool use_dt = false;  // decode on the TMA-fed persistent kernel (items cover all kv heads)
     int32_t num_ditems = 0, num_pitems = 0, num_groups = 0, num_parts = 0;
     void *d_ws = nullptr;
     size_t ws_bytes = 0;
@@ -195,6 +196,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->bt_width = width;
     pl->num_sms = sms;
     pl->flags = o.flags;
+    pl->use_dt = decode_tma_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_kv_heads,
+                                      desc->num_q_heads / desc->num_kv_heads, bs);
     pl->use_tc = !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
                  prefill_tc_supported(desc->head_dim_qk, desc->head_dim_v, bs,
                                       desc->num_q_heads / desc->num_kv_heads);
@@ -205,23 +208,37 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     std::vector<PrefillItem> pitems;
     std::vector<std::pair<int64_t, int32_t>> pcost;  // (cost, index) for LPT order
 
-    // decode split length: about 4 waves of 2 CTAs per SM over the decode keys
+    // decode split length: about 3 waves of 2 CTAs per SM over the decode work
+    // (a TMA decode item streams every kv head of its keys)
     int64_t dec_keys = 0;
     for (int32_t s = 0; s < num_seqs; ++s)
-        if (phase[s] == 1) dec_keys += static_cast<int64_t>(context_len[s]) * desc->num_kv_heads;
+        if (phase[s] == 1)
+            dec_keys += static_cast<int64_t>(context_len[s]) * (pl->use_dt ? 1 : desc->num_kv_heads);
     int32_t split = o.decode_split_keys;
     if (split == 0) {
-        const int64_t target = 8LL * sms;
+        const int64_t target = 6LL * sms;
         int64_t sk = (dec_keys + target - 1) / std::max<int64_t>(target, 1);
         sk = (sk + 63) / 64 * 64;
-        split = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(sk, 256), 4096));
+        split = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(sk, pl->use_dt ? 128 : 256), 4096));
     }
 
     int32_t qs = 0, parts = 0, groups = 0;
     for (int32_t s = 0; s < num_seqs; ++s) {
         seqs[s] = SeqInfo{qs, query_len[s], context_len[s], s};
         const int32_t q = query_len[s], c = context_len[s];
-        if (phase[s] == 1) {
+        if (phase[s] == 1 && pl->use_dt) {
+            // items over all kv heads; one merge counter per (sequence, kv head)
+            const int32_t sk = std::max(split, (c + 255 * 64) / (256 * 64) * 64);
+            const int32_t ns = (c + sk - 1) / sk;
+            const int32_t grp = groups;
+            groups += desc->num_kv_heads;
+            const int32_t base = ns > 1 ? parts : 0;
+            if (ns > 1) parts += ns;
+            for (int32_t sp = 0; sp < ns; ++sp) {
+                const int32_t kb = sp * sk, ke = std::min(c, kb + sk);
+                ditems.push_back(DecodeItem{s, 0, kb, ke, sp, ns, base, grp / desc->num_kv_heads});
+            }
+        } else if (phase[s] == 1) {
             const int32_t ns = (c + split - 1) / split;
             for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh) {
                 const int32_t grp = groups++;
@@ -281,10 +298,11 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
     const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
-    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 4, 256);  // err + work queue
+    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
     const size_t meta_bytes = off;
-    const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * G, 256);
-    const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * G * desc->head_dim_v, 256);
+    const int32_t part_rows = pl->use_dt ? desc->num_q_heads : G;  // query heads per partial
+    const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows, 256);
+    const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows * desc->head_dim_v, 256);
     pl->ws_bytes = off;
 
     if (cudaMalloc(&pl->d_ws, pl->ws_bytes) != cudaSuccess) {
@@ -371,7 +389,8 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
 
-    int rc = launch_decode_mma(p, stream);
+    int rc = pl->use_dt ? launch_decode_tma(p, stream)
+                        : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
     return pl->use_tc ? launch_prefill_tc(p, stream) : launch_prefill_mma(p, stream);
 }
@@ -383,7 +402,7 @@ int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
     int32_t v = 0;
     if (cudaMemcpy(&v, pl->d_err, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return FNPU_ECUDA;
     if (v != 0) {
-        const int32_t zero[4] = {0, 0, 0, 0};  // also resets the persistent work queue
+        const int32_t zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // also resets the persistent work queues
         if (cudaMemcpy(pl->d_err, zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
             return FNPU_ECUDA;
         return FNPU_EDEVICE_TIMEOUT;

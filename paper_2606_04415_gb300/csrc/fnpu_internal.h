@@ -8,10 +8,11 @@
 
 namespace fnpu {
 
-// One decode split item: keys [key_begin, key_end) of sequence `seq` for kv
-// head `kvh`, all G query heads of that group at the sequence's single query
-// position. Splits of one (seq, kvh) group share `group` (their merge counter)
-// and write partial results to scratch rows part_base + split.
+// One decode split item: keys [key_begin, key_end) of sequence `seq` at the
+// sequence's single query position, for kv head `kvh` and its G query heads
+// (per-head kernel) or for every kv head (all-heads kernel, kvh = 0). Splits
+// of one group share `group` (their merge counter) and write partial results
+// to scratch rows part_base + split.
 struct DecodeItem {
     int32_t seq, kvh, key_begin, key_end;
     int32_t split, num_splits, part_base, group;
@@ -60,7 +61,7 @@ struct AttnParams {
     const PrefillItem *pitems;
     int32_t num_pitems;
     int32_t *err;           // device error flag of the plan
-    int32_t *sched;         // [2] persistent work queue: next item, finished CTAs
+    int32_t *sched;         // persistent work queues: [0..1] prefill, [2..3] decode (next item, finished CTAs)
 };
 
 // Record a failed CUDA call for fnpu_last_cuda_error(); returns FNPU_ECUDA.
@@ -77,6 +78,8 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
                      void *stream);
 int read_and_clear_global_error(void *stream, int *flag);
 int launch_decode_mma(const AttnParams &p, void *stream);
+int launch_decode_tma(const AttnParams &p, void *stream);
+bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_prefill_mma(const AttnParams &p, void *stream);
 int launch_prefill_tc(const AttnParams &p, void *stream);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);

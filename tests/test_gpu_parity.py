@@ -248,3 +248,17 @@ def test_tc_and_mma_prefill_agree_on_coloc():
     a = _step(batch).results()
     b = _step(batch, flags=NO_TC).results()
     assert np.abs(a[0] - b[0]).max() <= O_TOL and np.abs(a[1] - b[1]).max() <= LSE_TOL
+
+
+@pytest.mark.parametrize("split", [0, 64, 192])
+@pytest.mark.parametrize("bs", [16, 32, 64])
+def test_decode_four_kv_heads_edges(bs, split):
+    """Hkv = 4 decodes (the TMA-fed decode kernel): contexts shorter than a
+    stage, not on stage or block edges, and several split lengths."""
+    sh = W.Shape(28, 4, 128, 128, bs, False)
+    ctx = [1, 2, 15, 16, 17, 63, 64, 65, 300, 1000, 2049]
+    rng = np.random.default_rng(7 * bs + split)
+    batch = W.build_batch(sh, [1] * len(ctx), ctx, [1] * len(ctx), rng, name="dec4")
+    st = _step(batch, split=split)
+    out, lse = st.results()
+    _compare(batch, out, lse)
