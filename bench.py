@@ -45,9 +45,15 @@ L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 def _flush_l2(wbuf, rbuf):
     """Evict L2 between timed steps: write a buffer larger than L2, then read
     another one so that L2 is left holding clean lines (otherwise the timed
-    kernel would pay for writing back ~126 MB of dirty flush data)."""
+    kernel would pay for writing back ~126 MB of dirty flush data). A short
+    device-side sleep follows, so that the host has queued the timed step's
+    launches before the device reaches them: the device-timed region then
+    measures kernel execution, not host enqueue latency (that is what the
+    end-to-end figure covers)."""
+    import torch
     wbuf.zero_()
     rbuf.sum()
+    torch.cuda._sleep(200_000)
 
 
 def _peaks():

@@ -1,27 +1,32 @@
-// Decode split-KV attention fed by TMA through an mbarrier pipeline
+// Decode split-KV attention fed by TMA through an mbarrier ring
 // (Hkv = 4 kv heads, d = 64 or 128, G <= 8 query heads per kv head, block
 // size a multiple of 16).
 //
-// Decode is bound by KV-cache reads (Sec. 1, Sec. 3.3, Fig. 2), so the kernel
-// is organised around keeping HBM busy:
-//   * persistent CTAs (two per SM) take items -- a sequence's key range,
-//     longest first -- from an atomic queue (the last CTA resets it);
-//   * one producer warp streams 16-key stages of K and V for all four kv
-//     heads (for Qwen one contiguous 16 KB slot run per stage and tensor) with
-//     four TMA boxes per stage into a 3-stage ring. The tensor map lists the
-//     slot dimension before the kv-head dimension, so a box lands head-major
-//     (16 consecutive slots of one head form 16 rows) and the 128-byte swizzle
-//     is keyed by the slot: ldmatrix over eight consecutive slots of one head
-//     is conflict-free;
-//   * four compute warps, one per kv head, run the GQA-packed mma.sync scheme
-//     independently (S^T = K Q^T with 16 keys in M and the G query heads in
-//     N; P^T by movmatrix; O^T += V^T P^T) and release a stage with one
-//     mbarrier arrival each -- no block-wide barrier per stage;
+// Decode is bound by KV-cache reads (Sec. 1, Sec. 3.3, Fig. 2). The kernel is
+// kept small -- four warps, at most 128 registers a thread, 64 KB of shared
+// memory for d = 128 -- so that up to three CTAs share an SM and a few SMs
+// alone can stream decode work while the others run prefill (Sec. 3.4).
+//   * Persistent CTAs take items -- a sequence's key range, longest first --
+//     from an atomic queue two items ahead of use (the last CTA out resets it);
+//     the next item's descriptor, block ids and query are loaded during the
+//     current item, so an item boundary costs no memory round trip.
+//   * A 2-stage ring of 16-key stages holds K and V of all four kv heads. Warp
+//     0 issues the TMA copies of the stage after the one it is about to read:
+//     four boxes of 16 slots x 4 heads x 64 columns for d = 128. The tensor map
+//     lists the slot dimension before the kv-head dimension, so a box lands
+//     head-major (16 consecutive slots of one head form 16 rows) and the
+//     128-byte swizzle is keyed by the slot: ldmatrix over eight consecutive
+//     slots of one head is conflict-free.
+//   * Each warp owns one kv head and runs the GQA-packed mma.sync scheme
+//     (S^T = K Q^T with the 16 keys in M and the G query heads in N; P^T by
+//     movmatrix; O^T += V^T P^T), releasing a stage with one mbarrier arrival.
 //   * V rows past the item's keys are zeroed by their warp before the PV
-//     product, so stale slots never reach it;
-//   * each warp writes its kv head's partial result; the last split of a
-//     (sequence, kv head) to finish merges all splits (atomic counter, no
-//     waiting).
+//     product, so stale slots never reach it.
+//   * A split writes its partial result (Eq. 1 restricted to its keys, with
+//     its log-sum-exp); the last split of a (sequence, kv head) to finish
+//     merges all of them. The release fence and the counter update of an item
+//     are deferred to the second stage of the next item, when the partial
+//     stores have long completed, and a merge they trigger to the end of it.
 // Every mbarrier wait is bounded and raises the plan's error flag on timeout.
 #include <math.h>
 
@@ -35,9 +40,9 @@ namespace {
 
 constexpr int kHkv = 4;
 constexpr int kKeys = 16;        // keys per stage
-constexpr int kStages = 3;
-constexpr int kCompute = 4;      // compute warps = kv heads
-constexpr int kThreads = 32 * (kCompute + 1);
+constexpr int kStages = 2;
+constexpr int kWarps = 4;        // one per kv head
+constexpr int kThreads = 32 * kWarps;
 constexpr int kHalfBytes = kHkv * kKeys * 128;  // all heads, one 64-column half
 
 template <int D>
@@ -45,9 +50,10 @@ struct DtCfg {
     static constexpr int kTileBytes = (D / 64) * kHalfBytes;  // K or V of one stage
     static constexpr int kStageBytes = 2 * kTileBytes;
     static constexpr int kBarOff = kStages * kStageBytes;
-    // full[S] empty[S] itemfull[2] itemempty[2]
-    static constexpr int kNumBars = 2 * kStages + 4;
-    static constexpr int kSmemBytes = 1024 + kBarOff + 8 * kNumBars + 16;
+    // full[S] empty[S] itemdone[2]
+    static constexpr int kNumBars = 2 * kStages + 2;
+    // + item ring [4] and the abort flag
+    static constexpr int kSmemBytes = kBarOff + 8 * kNumBars + 32;
 };
 
 struct DtMaps {
@@ -60,35 +66,72 @@ __device__ __forceinline__ uint32_t dt_off(int slot, int head, int chunk) {
                                  (((chunk & 7) ^ (slot & 7)) << 4));
 }
 
+// What a warp keeps of one item.
+struct DtGeo {
+    int t;          // query token
+    int bt_row;
+    int kb, ke;     // keys [kb, ke)
+    int split, ns, part_base, group;
+};
+
 template <int D>
-__global__ void __launch_bounds__(kThreads, 2)
+__device__ __forceinline__ void load_q(const AttnParams &p, int t, int head, int g8, int c,
+                                       uint32_t (&qb)[D / 16][2]) {
+    const __nv_bfloat16 *qrow = static_cast<const __nv_bfloat16 *>(p.q) +
+                                (static_cast<int64_t>(t) * p.num_q_heads + head * p.group) * D;
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        if (g8 < p.group) {
+            qb[kk][0] = __ldg(reinterpret_cast<const uint32_t *>(qrow + g8 * D + kk * 16 + 2 * c));
+            qb[kk][1] = __ldg(reinterpret_cast<const uint32_t *>(qrow + g8 * D + kk * 16 + 8 + 2 * c));
+        } else {
+            qb[kk][0] = qb[kk][1] = 0u;
+        }
+    }
+}
+
+// block ids of the item's blocks, relative block `lane` in lane `lane`
+__device__ __forceinline__ int load_blk_lane(const AttnParams &p, const DtGeo &g, int lane) {
+    const int b0 = g.kb / p.block_size;
+    const int nblk = (g.ke - 1) / p.block_size - b0 + 1;
+    return lane < nblk ? __ldg(p.block_table + static_cast<int64_t>(g.bt_row) * p.bt_stride + b0 + lane) : 0;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 4)
     decode_tma_kernel(const AttnParams p, const __grid_constant__ DtMaps maps) {
     using Cfg = DtCfg<D>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    extern __shared__ __align__(1024) uint8_t smem[];
     const uint32_t s_base = smem_u32(smem);
     const uint32_t s_bars = s_base + Cfg::kBarOff;
     auto FULL = [&](int s) { return s_bars + 8 * s; };
     auto EMPTY = [&](int s) { return s_bars + 8 * (kStages + s); };
-    auto ITEMFULL = [&](int k) { return s_bars + 8 * (2 * kStages + k); };
-    auto ITEMEMPTY = [&](int k) { return s_bars + 8 * (2 * kStages + 2 + k); };
-    uint8_t *misc = smem + Cfg::kBarOff + 8 * Cfg::kNumBars;
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc);
-    volatile int *item_slot = reinterpret_cast<volatile int *>(misc + 4);  // [2]
+    auto ITEMDONE = [&](int b) { return s_bars + 8 * (2 * kStages + b); };
+    int *ring = reinterpret_cast<int *>(smem + Cfg::kBarOff + 8 * Cfg::kNumBars);  // [4]
+    volatile int *abort_flag = ring + 4;
     int *sched = p.sched + 2;  // this kernel's work queue: next item, finished CTAs
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int n_items = p.num_ditems;
+    if ((s_base & 1023u) != 0) {  // the swizzled tiles need 1024-byte alignment
+        if (tid == 0) atomicOr(p.err, 2);
+        return;
+    }
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(FULL(s), 1);
-            tc::mbar_init(EMPTY(s), kCompute);
+            tc::mbar_init(EMPTY(s), kWarps);
         }
-        for (int k = 0; k < 2; ++k) {
-            tc::mbar_init(ITEMFULL(k), 1);
-            tc::mbar_init(ITEMEMPTY(k), kCompute);
-        }
+        tc::mbar_init(ITEMDONE(0), kWarps);
+        tc::mbar_init(ITEMDONE(1), kWarps);
+        ring[0] = atomicAdd(sched, 1);
+        ring[1] = atomicAdd(sched, 1);
         *abort_flag = 0;
         tc::fence_mbar_init();
+    }
+    if (warp == 0 && lane == 0) {
+        tc::prefetch_tmap(&maps.k);
+        tc::prefetch_tmap(&maps.v);
     }
     __syncthreads();
 
@@ -100,87 +143,178 @@ __global__ void __launch_bounds__(kThreads, 2)
         atomicOr(p.err, 1);
         return false;
     };
+    auto geo_of = [&](const DecodeItem &it, const SeqInfo &si) {
+        DtGeo g;
+        g.t = si.q_start;
+        g.bt_row = si.bt_row;
+        g.kb = it.key_begin;
+        g.ke = it.key_end;
+        g.split = it.split;
+        g.ns = it.num_splits;
+        g.part_base = it.part_base;
+        g.group = it.group;
+        return g;
+    };
 
-    if (warp == kCompute) {
-        // ------------------------------------------------ scheduler + producer
-        if (lane == 0) {
-            tc::prefetch_tmap(&maps.k);
-            tc::prefetch_tmap(&maps.v);
-        }
-        const int bs = p.block_size;
-        int g = 0;  // stages issued so far
-        for (int k = 0;; ++k) {
-            int idx = 0;
-            if (lane == 0) idx = atomicAdd(sched, 1);
-            idx = __shfl_sync(0xffffffffu, idx, 0);
-            const int slot = k & 1;
-            if (k >= 2 && !wait(ITEMEMPTY(slot), ((k >> 1) - 1) & 1)) break;
-            if (lane == 0) {
-                item_slot[slot] = idx < p.num_ditems ? idx : -1;
-                tc::mbar_arrive(ITEMFULL(slot));
-            }
-            if (idx >= p.num_ditems) break;
-            const DecodeItem it = p.ditems[idx];
-            const SeqInfo si = p.seqs[it.seq];
-            const int32_t *bt = p.block_table + static_cast<int64_t>(si.bt_row) * p.bt_stride;
-            const int ntiles = (it.key_end - it.key_begin + kKeys - 1) / kKeys;
-            // block id of the next stage, loaded one stage ahead
-            int blk_next = __ldg(bt + it.key_begin / bs);
-            bool ok = true;
-            for (int i = 0; i < ntiles; ++i, ++g) {
-                const int st = g % kStages;
-                const int key0 = it.key_begin + i * kKeys;
-                const int blk = __shfl_sync(0xffffffffu, blk_next, 0);
-                if (i + 1 < ntiles) blk_next = __ldg(bt + (key0 + kKeys) / bs);
-                if (g >= kStages && !wait(EMPTY(st), ((g / kStages) - 1) & 1)) { ok = false; break; }
-                const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
-                const int slot0 = __shfl_sync(0xffffffffu, key0 % bs, 0);
-                tc::mbar_arrive_expect_tx_warp(FULL(st), Cfg::kStageBytes);
+    const int head = warp;
+    const int g8 = lane >> 2, c = lane & 3;
+    const int lj = lane >> 3, lr = lane & 7;
+    const int G = p.group;
+    const int Hq = p.num_q_heads;
+    const int bs = p.block_size;
+    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
+
+    // issue stage `j` of item `g` into ring position `gs` (warp 0, whole warp)
+    auto issue = [&](const DtGeo &g, int j, int blk_lane, int gs) -> bool {
+        const int st = gs % kStages;
+        if (gs >= kStages && !wait(EMPTY(st), ((gs / kStages) - 1) & 1)) return false;
+        const int key0 = g.kb + j * kKeys;
+        const int rel = key0 / bs - g.kb / bs;
+        int blk = __shfl_sync(0xffffffffu, blk_lane, rel & 31);
+        if (rel >= 32) blk = __ldg(p.block_table + static_cast<int64_t>(g.bt_row) * p.bt_stride + key0 / bs);
+        const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
+        tc::mbar_arrive_expect_tx_warp(FULL(st), Cfg::kStageBytes);
 #pragma unroll
-                for (int h = 0; h < D / 64; ++h) {
-                    tc::tma_load_4d_warp(sK + h * kHalfBytes, &maps.k, FULL(st), h * 64, slot0, 0, blk);
-                    tc::tma_load_4d_warp(sV + h * kHalfBytes, &maps.v, FULL(st), h * 64, slot0, 0, blk);
+        for (int h = 0; h < D / 64; ++h) {
+            tc::tma_load_4d_warp(sK + h * kHalfBytes, &maps.k, FULL(st), h * 64, key0 % bs, 0, blk);
+            tc::tma_load_4d_warp(sV + h * kHalfBytes, &maps.v, FULL(st), h * 64, key0 % bs, 0, blk);
+        }
+        return true;
+    };
+
+    // merge of the splits of (sequence of token t, this kv head), by the last split
+    auto merge = [&](int t, int ns, int base) {
+        float M[8], L[8];
+#pragma unroll
+        for (int h = 0; h < 8; ++h) { M[h] = -INFINITY; L[h] = 0.f; }
+        for (int sp = lane; sp < ns; sp += 32) {
+            const float *pl = p.part_lse + static_cast<int64_t>(base + sp) * Hq + head * G;
+#pragma unroll
+            for (int h = 0; h < 8; ++h)
+                if (h < G) M[h] = fmaxf(M[h], __ldcg(pl + h));
+        }
+#pragma unroll
+        for (int h = 0; h < 8; ++h)
+#pragma unroll
+            for (int o2 = 16; o2 > 0; o2 >>= 1) M[h] = fmaxf(M[h], __shfl_xor_sync(0xffffffffu, M[h], o2));
+        for (int sp = lane; sp < ns; sp += 32) {
+            const float *pl = p.part_lse + static_cast<int64_t>(base + sp) * Hq + head * G;
+#pragma unroll
+            for (int h = 0; h < 8; ++h)
+                if (h < G) L[h] += fast_exp2(__ldcg(pl + h) - M[h]);
+        }
+#pragma unroll
+        for (int h = 0; h < 8; ++h)
+#pragma unroll
+            for (int o2 = 16; o2 > 0; o2 >>= 1) L[h] += __shfl_xor_sync(0xffffffffu, L[h], o2);
+        if (lane < D / 4) {
+            float4 acc[8];
+#pragma unroll
+            for (int h = 0; h < 8; ++h) acc[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
+#pragma unroll 2
+            for (int sp = 0; sp < ns; ++sp) {
+                const int64_t row = static_cast<int64_t>(base + sp) * Hq + head * G;
+#pragma unroll
+                for (int h = 0; h < 8; ++h) {
+                    if (h < G) {
+                        const float w = fast_exp2(__ldcg(p.part_lse + row + h) - M[h]);
+                        const float4 v = __ldcg(po + (row + h) * (D / 4) + lane);
+                        acc[h].x += w * v.x; acc[h].y += w * v.y; acc[h].z += w * v.z; acc[h].w += w * v.w;
+                    }
                 }
             }
-            if (!ok) break;
-        }
-    } else {
-        // ----------------------------------------- compute warp = one kv head
-        const int head = warp;
-        const int g8 = lane >> 2, c = lane & 3;
-        const int lj = lane >> 3, lr = lane & 7;
-        const int G = p.group;
-        const int Hq = p.num_q_heads;
-        int gs = 0;  // stages consumed so far
-        for (int k = 0;; ++k) {
-            const int slot = k & 1;
-            if (!wait(ITEMFULL(slot), (k >> 1) & 1)) break;
-            const int idx = __shfl_sync(0xffffffffu, item_slot[slot], 0);
-            if (idx < 0) break;
-            const DecodeItem it = p.ditems[idx];
-            const SeqInfo si = p.seqs[it.seq];
-            const int t = si.q_start;
-            const __nv_bfloat16 *qrow = static_cast<const __nv_bfloat16 *>(p.q) +
-                                        (static_cast<int64_t>(t) * Hq + head * G) * D;
-            uint32_t qb[D / 16][2];
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-                if (g8 < G) {
-                    qb[kk][0] = __ldg(reinterpret_cast<const uint32_t *>(qrow + g8 * D + kk * 16 + 2 * c));
-                    qb[kk][1] = __ldg(reinterpret_cast<const uint32_t *>(qrow + g8 * D + kk * 16 + 8 + 2 * c));
-                } else {
-                    qb[kk][0] = qb[kk][1] = 0u;
+            for (int h = 0; h < 8; ++h) {
+                if (h < G) {
+                    const float il = 1.f / L[h];
+                    uint2 pk;
+                    pk.x = pack_bf16x2(acc[h].x * il, acc[h].y * il);
+                    pk.y = pack_bf16x2(acc[h].z * il, acc[h].w * il);
+                    *reinterpret_cast<uint2 *>(out + (static_cast<int64_t>(t) * Hq + head * G + h) * D + lane * 4) = pk;
                 }
             }
-            const int nkeys = it.key_end - it.key_begin;
-            const int ntiles = (nkeys + kKeys - 1) / kKeys;
+        }
+        if (lane < G) {
+            float Ml = M[0], Ll = L[0];
+#pragma unroll
+            for (int h = 1; h < 8; ++h)
+                if (lane == h) { Ml = M[h]; Ll = L[h]; }
+            p.lse[static_cast<int64_t>(t) * Hq + head * G + lane] = (Ml + log2f(Ll)) * kLn2;
+        }
+    };
+
+    // A finished split's counter update waits until its partial stores have
+    // completed (a stage into the next item); a merge it triggers runs at the
+    // end of that next item, when the accumulators are free.
+    bool pend = false, mrg = false;
+    int pend_t = 0, pend_ns = 0, pend_base = 0, pend_group = 0;
+    auto settle = [&]() {
+        if (!pend) return;
+        pend = false;
+        __threadfence();  // this warp's partial stores before the counter update
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) last = atomicAdd(p.counters + pend_group * kHkv + head, 1) == pend_ns - 1;
+        mrg = __shfl_sync(0xffffffffu, last, 0) != 0;
+    };
+    auto merge_if_last = [&]() {
+        if (!mrg) return;
+        mrg = false;
+        __threadfence();
+        merge(pend_t, pend_ns, pend_base);
+        if (lane == 0) p.counters[pend_group * kHkv + head] = 0;  // ready for the next run
+    };
+
+    int idx = ring[0];
+    if (idx < n_items) {
+        DtGeo cur;
+        {
+            const DecodeItem it = p.ditems[idx];
+            cur = geo_of(it, p.seqs[it.seq]);
+        }
+        uint32_t qb[D / 16][2];
+        load_q<D>(p, cur.t, head, g8, c, qb);
+        int blk_lane = warp == 0 ? load_blk_lane(p, cur, lane) : 0;
+        bool ok = true;
+        if (warp == 0) ok = issue(cur, 0, blk_lane, 0);
+        int g = 0;  // ring position of the current item's first stage
+        for (int k = 0; ok; ++k) {
+            const int ntiles = (cur.ke - cur.kb + kKeys - 1) / kKeys;
+            const int idx_n = ring[(k + 1) & 3];
+            const bool has_next = idx_n < n_items;
+            int a_next = 0;
+            if (warp == 0 && lane == 0) a_next = atomicAdd(sched, 1);  // the item after next
+            DecodeItem nit{};
+            if (has_next) nit = p.ditems[idx_n];
+            SeqInfo nsi{};
+            DtGeo nxt{};
+            uint32_t qn[D / 16][2];
+            int blk_lane_n = 0;
+
             float o[D / 16][4];
 #pragma unroll
             for (int mt = 0; mt < D / 16; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
             float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-            bool ok = true;
-            for (int i = 0; i < ntiles; ++i, ++gs) {
+            const int nkeys = cur.ke - cur.kb;
+            bool nready = false;
+            for (int i = 0; i < ntiles; ++i) {
+                const int gs = g + i;
                 const int st = gs % kStages;
+                // the next item: its sequence row after stage 0, its block ids
+                // and query from stage 2 on (or before its first stage is issued)
+                if (has_next && !nready && (i == 2 || i == ntiles - 1)) {
+                    if (i == 0) nsi = p.seqs[nit.seq];
+                    nxt = geo_of(nit, nsi);
+                    load_q<D>(p, nxt.t, head, g8, c, qn);
+                    if (warp == 0) blk_lane_n = load_blk_lane(p, nxt, lane);
+                    nready = true;
+                }
+                if (warp == 0) {
+                    if (i + 1 < ntiles) ok = issue(cur, i + 1, blk_lane, gs + 1);
+                    else if (has_next) ok = issue(nxt, 0, blk_lane_n, gs + 1);
+                    if (!ok) break;
+                }
                 if (!wait(FULL(st), (gs / kStages) & 1)) { ok = false; break; }
                 const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
                 const int nv = nkeys - i * kKeys;  // valid keys in this stage (>= 1)
@@ -234,6 +368,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                 if (tail) tc::fence_proxy_async_smem();  // order the zeroing before the next TMA write
                 __syncwarp();
                 tc::mbar_arrive_warp(EMPTY(st));
+                if (i == 0 && has_next && !nready) nsi = p.seqs[nit.seq];
+                if (i == 1) settle();  // the previous item's counter, now that its stores are done
             }
             if (!ok) break;
             l0 += __shfl_xor_sync(0xffffffffu, l0, 4);
@@ -244,28 +380,28 @@ __global__ void __launch_bounds__(kThreads, 2)
             l1 += __shfl_xor_sync(0xffffffffu, l1, 16);
             const float inv0 = 1.f / l0, inv1 = 1.f / l1;
             const int h0 = 2 * c, h1 = 2 * c + 1;  // this lane's query heads within the group
-            __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
-            if (it.num_splits == 1) {
+            settle();  // (the previous item, if this one had a single stage)
+            if (cur.ns == 1) {
 #pragma unroll
                 for (int mt = 0; mt < D / 16; ++mt) {
                     const int d0 = mt * 16 + g8;
                     if (h0 < G) {
-                        __nv_bfloat16 *r = out + (static_cast<int64_t>(t) * Hq + head * G + h0) * D;
+                        __nv_bfloat16 *r = out + (static_cast<int64_t>(cur.t) * Hq + head * G + h0) * D;
                         r[d0] = __float2bfloat16_rn(o[mt][0] * inv0);
                         r[d0 + 8] = __float2bfloat16_rn(o[mt][2] * inv0);
                     }
                     if (h1 < G) {
-                        __nv_bfloat16 *r = out + (static_cast<int64_t>(t) * Hq + head * G + h1) * D;
+                        __nv_bfloat16 *r = out + (static_cast<int64_t>(cur.t) * Hq + head * G + h1) * D;
                         r[d0] = __float2bfloat16_rn(o[mt][1] * inv1);
                         r[d0 + 8] = __float2bfloat16_rn(o[mt][3] * inv1);
                     }
                 }
                 if (g8 == 0) {
-                    if (h0 < G) p.lse[static_cast<int64_t>(t) * Hq + head * G + h0] = (m0 + log2f(l0)) * kLn2;
-                    if (h1 < G) p.lse[static_cast<int64_t>(t) * Hq + head * G + h1] = (m1 + log2f(l1)) * kLn2;
+                    if (h0 < G) p.lse[static_cast<int64_t>(cur.t) * Hq + head * G + h0] = (m0 + log2f(l0)) * kLn2;
+                    if (h1 < G) p.lse[static_cast<int64_t>(cur.t) * Hq + head * G + h1] = (m1 + log2f(l1)) * kLn2;
                 }
             } else {
-                const int64_t part = it.part_base + it.split;
+                const int64_t part = cur.part_base + cur.split;
 #pragma unroll
                 for (int mt = 0; mt < D / 16; ++mt) {
                     const int d0 = mt * 16 + g8;
@@ -284,47 +420,30 @@ __global__ void __launch_bounds__(kThreads, 2)
                     if (h0 < G) p.part_lse[part * Hq + head * G + h0] = m0 + log2f(l0);
                     if (h1 < G) p.part_lse[part * Hq + head * G + h1] = m1 + log2f(l1);
                 }
-                // the last split of this (sequence, kv head) merges all splits
-                __threadfence();
-                __syncwarp();
-                int last = 0;
-                if (lane == 0) last = atomicAdd(p.counters + it.group * kHkv + head, 1) == it.num_splits - 1;
-                last = __shfl_sync(0xffffffffu, last, 0);
-                if (last) {
-                    __threadfence();
-                    const int ns = it.num_splits;
-                    const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
-                    for (int hg = 0; hg < G; ++hg) {
-                        const int qh = head * G + hg;
-                        float M = -INFINITY;
-                        for (int sp = lane; sp < ns; sp += 32)
-                            M = fmaxf(M, __ldcg(p.part_lse + static_cast<int64_t>(it.part_base + sp) * Hq + qh));
-                        for (int o2 = 16; o2 > 0; o2 >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o2));
-                        float L = 0.f;
-                        for (int sp = lane; sp < ns; sp += 32)
-                            L += fast_exp2(__ldcg(p.part_lse + static_cast<int64_t>(it.part_base + sp) * Hq + qh) - M);
-                        for (int o2 = 16; o2 > 0; o2 >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o2);
-                        if (lane < D / 4) {
-                            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-                            for (int sp = 0; sp < ns; ++sp) {
-                                const int64_t pr = it.part_base + sp;
-                                const float w = fast_exp2(__ldcg(p.part_lse + pr * Hq + qh) - M);
-                                const float4 v = __ldcg(po + (pr * Hq + qh) * (D / 4) + lane);
-                                acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
-                            }
-                            const float il = 1.f / L;
-                            uint2 pk;
-                            pk.x = pack_bf16x2(acc.x * il, acc.y * il);
-                            pk.y = pack_bf16x2(acc.z * il, acc.w * il);
-                            *reinterpret_cast<uint2 *>(out + (static_cast<int64_t>(t) * Hq + qh) * D + lane * 4) = pk;
-                        }
-                        if (lane == 0) p.lse[static_cast<int64_t>(t) * Hq + qh] = (M + log2f(L)) * kLn2;
-                    }
-                    if (lane == 0) p.counters[it.group * kHkv + head] = 0;  // ready for the next run
-                }
             }
-            tc::mbar_arrive_warp(ITEMEMPTY(slot));
+            merge_if_last();  // the previous item's merge, with this item's accumulators stored
+            if (cur.ns > 1) {
+                pend = true;
+                pend_t = cur.t;
+                pend_ns = cur.ns;
+                pend_base = cur.part_base;
+                pend_group = cur.group;
+            }
+            // publish the item after next, then step to the next item
+            if (warp == 0 && lane == 0) ring[(k + 2) & 3] = a_next;
+            __syncwarp();
+            tc::mbar_arrive_warp(ITEMDONE(k & 1));
+            if (!wait(ITEMDONE(k & 1), (k >> 1) & 1)) break;
+            if (!has_next) break;
+            g += ntiles;
+            cur = nxt;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) { qb[kk][0] = qn[kk][0]; qb[kk][1] = qn[kk][1]; }
+            blk_lane = blk_lane_n;
+        }
+        if (!*abort_flag) {
+            settle();
+            merge_if_last();
         }
     }
 
@@ -376,7 +495,7 @@ bool encode_slot_major_map(CUtensorMap *m, const void *base, int d, int hkv, int
 }
 
 template <int D>
-int launch_dt(const AttnParams &p, cudaStream_t st) {
+int launch_dt(const AttnParams &p, cudaStream_t st, int max_ctas) {
     using Cfg = DtCfg<D>;
     DtMaps maps;
     if (!encode_slot_major_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
@@ -384,10 +503,9 @@ int launch_dt(const AttnParams &p, cudaStream_t st) {
         return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled (decode)");
     FNPU_CUDA_TRY(cudaFuncSetAttribute(decode_tma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmemBytes));
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int grid = p.num_ditems < 2 * sms ? p.num_ditems : 2 * sms;
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(decode_tma_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                       cudaSharedmemCarveoutMaxShared));
+    const int grid = p.num_ditems < max_ctas ? p.num_ditems : max_ctas;
     decode_tma_kernel<D><<<grid, kThreads, Cfg::kSmemBytes, st>>>(p, maps);
     FNPU_CUDA_TRY(cudaGetLastError());
     return FNPU_OK;
@@ -399,12 +517,12 @@ bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size)
     return d_qk == d_v && (d_qk == 64 || d_qk == 128) && hkv == kHkv && group <= 8 && block_size % kKeys == 0;
 }
 
-int launch_decode_tma(const AttnParams &p, void *stream) {
+int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas) {
     if (p.num_ditems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     switch (p.head_dim_qk) {
-        case 64: return launch_dt<64>(p, st);
-        case 128: return launch_dt<128>(p, st);
+        case 64: return launch_dt<64>(p, st, max_ctas);
+        case 128: return launch_dt<128>(p, st, max_ctas);
         default: return FNPU_EUNSUPPORTED;
     }
 }

@@ -389,7 +389,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
 
-    int rc = pl->use_dt ? launch_decode_tma(p, stream)
+    int rc = pl->use_dt ? launch_decode_tma(p, stream, 3 * pl->num_sms)
                         : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
     return pl->use_tc ? launch_prefill_tc(p, stream) : launch_prefill_mma(p, stream);

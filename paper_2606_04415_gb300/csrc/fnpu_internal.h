@@ -78,7 +78,7 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
                      void *stream);
 int read_and_clear_global_error(void *stream, int *flag);
 int launch_decode_mma(const AttnParams &p, void *stream);
-int launch_decode_tma(const AttnParams &p, void *stream);
+int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas);
 bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_prefill_mma(const AttnParams &p, void *stream);
 int launch_prefill_tc(const AttnParams &p, void *stream);
