@@ -52,7 +52,8 @@ typedef enum {
     FNPU_EINVAL = -1,          /* bad argument; nothing was launched */
     FNPU_EUNSUPPORTED = -2,    /* valid but not implemented (head dims etc.) */
     FNPU_ECUDA = -3,           /* a CUDA runtime call failed */
-    FNPU_EDEVICE_TIMEOUT = -4, /* a bounded device-side wait gave up */
+    FNPU_EDEVICE_TIMEOUT = -4, /* a bounded device-side wait gave up, or a kernel
+                                  found its shared memory misaligned and did nothing */
     FNPU_ENOMEM = -5,          /* device or host allocation failed */
     FNPU_EDEVICE_RANGE = -6    /* a kernel met an out-of-range slot and skipped it */
 } fnpu_status;
@@ -141,7 +142,9 @@ int fnpu_mixed_attn_run(const fnpu_plan *plan, const void *q, const void *k_cach
                         const void *v_cache, void *out, float *lse, void *stream);
 
 /* Synchronise `stream`, then read and clear the plan's device error flag:
- * FNPU_OK, FNPU_EDEVICE_TIMEOUT or FNPU_ECUDA. */
+ * FNPU_OK, FNPU_EDEVICE_TIMEOUT or FNPU_ECUDA. After FNPU_EDEVICE_TIMEOUT the
+ * outputs of the failed run are undefined; the plan's work queues and split
+ * counters are reset, so the plan can be run again. */
 int fnpu_plan_check(const fnpu_plan *plan, void *stream);
 
 /* Synchronise `stream`, then read and clear the library-wide device error

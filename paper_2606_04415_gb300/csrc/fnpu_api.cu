@@ -41,6 +41,10 @@ struct fnpu_plan {
     int32_t *d_err = nullptr;
     float *d_part_lse = nullptr;
     float *d_part_o = nullptr;
+    int32_t *d_pcounters = nullptr;
+    float *d_ppart_lse = nullptr;
+    float *d_ppart_o = nullptr;
+    int32_t num_pparts = 0, num_pgroups = 0;
 };
 
 namespace fnpu {
@@ -56,6 +60,77 @@ int cuda_fail(cudaError_t e, const char *where) {
 namespace {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Two packed Q tiles of one kv head (the tcgen05 prefill unit) before its key
+// range is split.
+struct TcUnit {
+    int32_t seq, kvh, r0, rows;
+    int32_t ntiles;     // 64-key tiles its rows can see
+    int32_t max_start;  // last tile a split may start at: every row must see a key of every split
+};
+
+// Cost model of a prefill work item in units of one 64-key tile of both Q
+// tiles: switching items (loading Q, draining the pipeline, the epilogue) and,
+// for a split item, writing its partial result and the merge.
+constexpr int64_t kTcItemCost = 2;
+constexpr int64_t kTcMergeCost = 3;
+
+// First tile of split j of n over ntiles tiles (split n is the end).
+int32_t split_bound(int32_t ntiles, int32_t n, int32_t j) {
+    return static_cast<int32_t>((static_cast<int64_t>(ntiles) * j) / n);
+}
+
+// Longest-processing-time-first makespan of `costs` (sorted descending) on m
+// workers.
+int64_t lpt_makespan(const std::vector<int64_t> &costs, int32_t m) {
+    std::vector<int64_t> heap(static_cast<size_t>(std::max(m, 1)), 0);  // min-heap of loads
+    auto cmp = [](int64_t a, int64_t b) { return a > b; };
+    for (int64_t c : costs) {
+        std::pop_heap(heap.begin(), heap.end(), cmp);
+        heap.back() += c;
+        std::push_heap(heap.begin(), heap.end(), cmp);
+    }
+    return *std::max_element(heap.begin(), heap.end());
+}
+
+// Number of key splits per unit. A persistent CTA per SM takes items longest
+// first, so the step lasts about as long as the LPT schedule of the items.
+// Splitting the largest units evens that schedule out but costs a partial
+// write and a merge, so the piece-size cap is chosen among a few candidates
+// by the modelled makespan.
+std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int32_t sms) {
+    int64_t total = 0, maxc = 0;
+    for (const TcUnit &u : units) {
+        total += u.ntiles;
+        maxc = std::max<int64_t>(maxc, u.ntiles);
+    }
+    std::vector<int64_t> caps = {maxc};
+    for (int k = 2; k <= 8; ++k) caps.push_back((maxc + k - 1) / k);
+    for (int j = 1; j <= 8; ++j) caps.push_back((total + static_cast<int64_t>(sms) * j - 1) / (static_cast<int64_t>(sms) * j));
+    std::vector<int32_t> best(units.size(), 1), ns(units.size(), 1);
+    int64_t best_span = -1;
+    std::vector<int64_t> costs;
+    for (int64_t cap : caps) {
+        if (cap < 8) continue;  // pieces shorter than this cost more than they balance
+        costs.clear();
+        for (size_t i = 0; i < units.size(); ++i) {
+            const TcUnit &u = units[i];
+            int32_t n = static_cast<int32_t>(std::min<int64_t>((u.ntiles + cap - 1) / cap, 16));
+            while (n > 1 && split_bound(u.ntiles, n, n - 1) > u.max_start) --n;
+            ns[i] = n;
+            for (int32_t j = 0; j < n; ++j)
+                costs.push_back(split_bound(u.ntiles, n, j + 1) - split_bound(u.ntiles, n, j) + kTcItemCost +
+                                (n > 1 ? kTcMergeCost : 0));
+        }
+        std::sort(costs.begin(), costs.end(), [](int64_t a, int64_t b) { return a > b; });
+        const int64_t span = lpt_makespan(costs, sms);
+        if (best_span < 0 || span < best_span) {
+            best_span = span;
+            best = ns;
+        }
+    }
+    return best;
+}
 
 bool shape_ok(const fnpu_attn_desc *d, int *status) {
     *status = FNPU_EINVAL;
@@ -207,6 +282,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     std::vector<DecodeItem> ditems;
     std::vector<PrefillItem> pitems;
     std::vector<std::pair<int64_t, int32_t>> pcost;  // (cost, index) for LPT order
+    std::vector<TcUnit> tc_units;
 
     // decode split length: about 3 waves of 2 CTAs per SM over the decode work
     // (a TMA decode item streams every kv head of its keys)
@@ -250,16 +326,15 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 }
             }
         } else if (pl->use_tc) {
-            // tcgen05 tiles: P positions x G heads of one kv head per tile
+            // tcgen05 tiles: two Q tiles of P positions x G heads of one kv
+            // head; their key splits are chosen once all tiles are known
             const int32_t prefix = c - q;
-            const int32_t P = prefill_tc_rows_per_item(G);
-            for (int32_t r0 = 0; r0 < q; r0 += P) {
-                const int32_t rows = std::min(P, q - r0);
-                for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh) {
-                    pcost.emplace_back(static_cast<int64_t>(prefix) + r0 + rows,
-                                       static_cast<int32_t>(pitems.size()));
-                    pitems.push_back(PrefillItem{s, kvh, r0, rows});
-                }
+            const int32_t P2 = prefill_tc_rows_per_item(G);
+            for (int32_t r0 = 0; r0 < q; r0 += P2) {
+                const int32_t rows = std::min(P2, q - r0);
+                const int32_t ntiles = (prefix + r0 + rows + 63) / 64;
+                for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh)
+                    tc_units.push_back(TcUnit{s, kvh, r0, rows, ntiles, (prefix + r0) / 64});
             }
         } else {
             const int32_t prefix = c - q;
@@ -268,11 +343,30 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 for (int32_t h = 0; h < desc->num_q_heads; ++h) {
                     pcost.emplace_back(static_cast<int64_t>(prefix) + r0 + rows,
                                        static_cast<int32_t>(pitems.size()));
-                    pitems.push_back(PrefillItem{s, h, r0, rows});
+                    pitems.push_back(PrefillItem{s, h, r0, rows, 0, 0, 0, 1, 0, 0, 0, 0});
                 }
             }
         }
         qs += query_len[s];
+    }
+    int32_t pparts = 0, pgroups = 0;
+    if (!tc_units.empty()) {
+        const std::vector<int32_t> ns = choose_prefill_splits(tc_units, sms);
+        for (size_t u = 0; u < tc_units.size(); ++u) {
+            const TcUnit &t = tc_units[u];
+            const int32_t n = ns[u];
+            const int32_t base = n > 1 ? pparts : 0, grp = n > 1 ? pgroups : 0;
+            if (n > 1) {
+                pparts += n;
+                pgroups += 1;
+            }
+            for (int32_t j = 0; j < n; ++j) {
+                const int32_t kb = split_bound(t.ntiles, n, j), ke = split_bound(t.ntiles, n, j + 1);
+                pcost.emplace_back(static_cast<int64_t>(ke - kb) + kTcItemCost + (n > 1 ? kTcMergeCost : 0),
+                                   static_cast<int32_t>(pitems.size()));
+                pitems.push_back(PrefillItem{t.seq, t.kvh, t.r0, t.rows, kb, ke, j, n, base, grp, 0, 0});
+            }
+        }
     }
     // longest prefill tiles first; decode items longest first as well
     std::stable_sort(pcost.begin(), pcost.end(),
@@ -290,6 +384,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->num_pitems = static_cast<int32_t>(pordered.size());
     pl->num_groups = groups;
     pl->num_parts = parts;
+    pl->num_pparts = pparts;
+    pl->num_pgroups = pgroups;
 
     // workspace: metadata (uploaded) then scratch (never read before written)
     size_t off = 0;
@@ -298,11 +394,14 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
     const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
+    const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
     const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
     const size_t meta_bytes = off;
     const int32_t part_rows = pl->use_dt ? desc->num_q_heads : G;  // query heads per partial
     const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows, 256);
     const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows * desc->head_dim_v, 256);
+    const size_t o_pplse = off; off = align_up(off + sizeof(float) * 256 * static_cast<size_t>(std::max(pparts, 1)), 256);
+    const size_t o_ppo = off; off = align_up(off + sizeof(float) * 256 * static_cast<size_t>(std::max(pparts, 1)) * desc->head_dim_v, 256);
     pl->ws_bytes = off;
 
     if (cudaMalloc(&pl->d_ws, pl->ws_bytes) != cudaSuccess) {
@@ -335,6 +434,9 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->d_err = reinterpret_cast<int32_t *>(d + o_err);
     pl->d_part_lse = reinterpret_cast<float *>(d + o_plse);
     pl->d_part_o = reinterpret_cast<float *>(d + o_po);
+    pl->d_pcounters = reinterpret_cast<int32_t *>(d + o_pcnt);
+    pl->d_ppart_lse = reinterpret_cast<float *>(d + o_pplse);
+    pl->d_ppart_o = reinterpret_cast<float *>(d + o_ppo);
     if (cudaMemcpyAsync(pl->d_ws, pl->h_stage, meta_bytes, cudaMemcpyHostToDevice,
                         static_cast<cudaStream_t>(stream)) != cudaSuccess) {
         cudaGetLastError();
@@ -386,6 +488,9 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.counters = pl->d_counters;
     p.pitems = pl->d_pitems;
     p.num_pitems = pl->num_pitems;
+    p.ppart_o = pl->d_ppart_o;
+    p.ppart_lse = pl->d_ppart_lse;
+    p.pcounters = pl->d_pcounters;
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
 
@@ -404,6 +509,11 @@ int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
     if (v != 0) {
         const int32_t zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // also resets the persistent work queues
         if (cudaMemcpy(pl->d_err, zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+            return FNPU_ECUDA;
+        // an aborted run can leave split-merge counters behind
+        if (cudaMemset(pl->d_counters, 0, sizeof(int32_t) * std::max(pl->num_groups, 1)) != cudaSuccess ||
+            cudaMemset(pl->d_pcounters, 0, sizeof(int32_t) * 8 * std::max(pl->num_pgroups, 1)) != cudaSuccess ||
+            cudaDeviceSynchronize() != cudaSuccess)
             return FNPU_ECUDA;
         return FNPU_EDEVICE_TIMEOUT;
     }

@@ -21,11 +21,18 @@ static_assert(sizeof(DecodeItem) == 32, "DecodeItem layout");
 
 // One prefill tile: query rows [row_begin, row_begin + rows) of sequence
 // `seq`'s chunk for query head `head` (the mma.sync path) or for kv head
-// `head` with all its query heads packed (the tcgen05 path).
+// `head` with all its query heads packed (the tcgen05 path). The tcgen05 path
+// may split the keys of a tile: the item then covers 64-key tiles
+// [kt_begin, kt_end) only, writes its partial result to scratch row
+// part_base + split and the last split of the tile to finish (merge counter
+// `group`) combines all num_splits of them. Unsplit items have
+// num_splits == 1 and cover every key their rows can see.
 struct PrefillItem {
     int32_t seq, head, row_begin, rows;
+    int32_t kt_begin, kt_end, split, num_splits;
+    int32_t part_base, group, pad0, pad1;
 };
-static_assert(sizeof(PrefillItem) == 16, "PrefillItem layout");
+static_assert(sizeof(PrefillItem) == 48, "PrefillItem layout");
 
 // Per-sequence metadata on the device.
 struct SeqInfo {
@@ -60,6 +67,9 @@ struct AttnParams {
     // prefill
     const PrefillItem *pitems;
     int32_t num_pitems;
+    float *ppart_o;         // fp32 split-prefill partials, per partial: [2 tiles][dv / 4][128 rows] float4
+    float *ppart_lse;       // fp32 [num_pparts, 2, 128] (log2 domain)
+    int32_t *pcounters;     // [num_pgroups, 8] one per softmax warp, zero between runs
     int32_t *err;           // device error flag of the plan
     int32_t *sched;         // persistent work queues: [0..1] prefill, [2..3] decode (next item, finished CTAs)
 };

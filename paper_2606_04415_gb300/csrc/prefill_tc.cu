@@ -70,7 +70,7 @@ struct TcCfg {
     // kfull[S] vfull[S] kempty[S] vempty[S] sfull[2] sfree[2] pfull[2][2] pvdone[2][2]
     // qfull qempty vzero itemfull[2] itemempty[2] drain[2]
     static constexpr int kNumBars = 4 * kStages + 12 + 9;
-    static constexpr int kSmemUsed = 1024 + kBarOff + 8 * kNumBars + 32;
+    static constexpr int kSmemUsed = kBarOff + 8 * kNumBars + 32;
     // at least 116 KB so that no two CTAs share an SM (each holds all 512 TMEM columns)
     static constexpr int kSmemBytes = kSmemUsed > 116 * 1024 ? kSmemUsed : 116 * 1024;
     static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
@@ -81,7 +81,8 @@ struct TcMaps {
 };
 
 struct ItemGeom {
-    int kvh, p0, rows, prefix, ctx, ntiles, q_start, bt_row;
+    int kvh, p0, rows, prefix, ctx, kt0, ntiles, q_start, bt_row;
+    int ns, split, pbase, cnt;  // key splits of the tile pair, this split, first partial, merge counter
     bool tail_fix;
 };
 
@@ -94,11 +95,15 @@ __device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
     g.rows = it.rows;
     g.prefix = si.ctx_len - si.q_len;
     g.ctx = si.ctx_len;
-    const int nkeys = g.prefix + it.row_begin + it.rows;  // keys 0 .. last position
-    g.ntiles = (nkeys + kKeys - 1) / kKeys;
+    g.kt0 = it.kt_begin;              // 64-key tiles [kt_begin, kt_end) of keys 0 .. last position
+    g.ntiles = it.kt_end - it.kt_begin;
     g.q_start = si.q_start;
     g.bt_row = si.bt_row;
-    g.tail_fix = g.ntiles * kKeys > g.ctx;
+    g.ns = it.num_splits;
+    g.split = it.split;
+    g.pbase = it.part_base;
+    g.cnt = it.group;
+    g.tail_fix = it.kt_end * kKeys > g.ctx;
     return g;
 }
 
@@ -106,8 +111,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_tc_kernel(const AttnParams p, const __grid_constant__ TcMaps maps) {
     using Cfg = TcCfg<D>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    extern __shared__ __align__(1024) uint8_t smem[];
     const uint32_t s_base = smem_u32(smem);
     const uint32_t s_bars = s_base + Cfg::kBarOff;
     auto KFULL = [&](int s) { return s_bars + 8 * s; };
@@ -131,6 +135,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = p.group;
     const int P = kRows / G;
+    if ((s_base & 1023u) != 0) {  // the swizzled tiles need 1024-byte alignment
+        if (tid == 0) atomicOr(p.err, 2);
+        return;
+    }
 
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -220,15 +228,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int nblk_seq = (it.ctx + bs - 1) / bs;
             // block ids of the next tile, one per lane, loaded a tile ahead so
             // that the TMA issue never waits on a block-table read
-            int blk_next = (lane < per_tile && lane < nblk_seq) ? __ldg(bt + lane) : 0;
+            const int b00 = it.kt0 * per_tile;
+            int blk_next = (lane < per_tile && b00 + lane < nblk_seq) ? __ldg(bt + b00 + lane) : 0;
             bool ok = true;
             for (int i = 0; i < it.ntiles; ++i, ++g) {
                 const int st = g % kStages;
                 const int blk_cur = blk_next;
-                const int jn = (i + 1) * per_tile + lane;
+                const int jn = b00 + (i + 1) * per_tile + lane;
                 blk_next = (i + 1 < it.ntiles && lane < per_tile && jn < nblk_seq) ? __ldg(bt + jn) : 0;
                 if (g >= kStages && !wait(is_k ? KEMPTY(st) : VEMPTY(st), ((g / kStages) - 1) & 1)) { ok = false; break; }
-                int nvalid = nblk_seq - i * per_tile;
+                int nvalid = nblk_seq - b00 - i * per_tile;
                 nvalid = nvalid < 0 ? 0 : (nvalid > per_tile ? per_tile : nvalid);
                 nvalid = __shfl_sync(0xffffffffu, nvalid, 0);
                 const uint32_t dst = s_base + st * Cfg::kStageBytes + (is_k ? 0 : Cfg::kTileBytes);
@@ -246,7 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!is_k && i == it.ntiles - 1 && it.tail_fix) {
                     // zero V rows of keys >= ctx (stale slots, unloaded blocks)
                     if (!wait(VFULL(st), (g / kStages) & 1)) { ok = false; break; }
-                    const int r0 = it.ctx - i * kKeys;
+                    const int r0 = it.ctx - (it.kt0 + i) * kKeys;
                     const int nrows = kKeys - r0;
                     for (int e = lane; e < nrows * 8 * (D / 64); e += 32) {
                         const int h = e / (nrows * 8), rem = e % (nrows * 8);
@@ -390,7 +399,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::mbar_arrive(SFREE(w));  // the S buffer may be overwritten now
                 // tiles that reach past the first row's position need the causal
                 // mask; all others are fully visible to every row of the tile
-                const int k0 = i * kKeys;
+                const int k0 = (it.kt0 + i) * kKeys;
                 const bool masked_tile = k0 + kKeys - 1 > min_pos;
                 float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
                 if (masked_tile) {
@@ -463,24 +472,108 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float inv = 1.f / l;
             uint4 *orow = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
                                                     (tok * p.num_q_heads + head) * D);
+            if (it.ns == 1) {
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
-                tc::tmem_wait_ld();
-                if (row_ok) {
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
+                    tc::tmem_wait_ld();
+                    if (row_ok) {
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        uint4 v;
-                        v.x = pack_bf16x2(__uint_as_float(o[8 * j + 0]) * inv, __uint_as_float(o[8 * j + 1]) * inv);
-                        v.y = pack_bf16x2(__uint_as_float(o[8 * j + 2]) * inv, __uint_as_float(o[8 * j + 3]) * inv);
-                        v.z = pack_bf16x2(__uint_as_float(o[8 * j + 4]) * inv, __uint_as_float(o[8 * j + 5]) * inv);
-                        v.w = pack_bf16x2(__uint_as_float(o[8 * j + 6]) * inv, __uint_as_float(o[8 * j + 7]) * inv);
-                        orow[c * 4 + j] = v;
+                        for (int j = 0; j < 4; ++j) {
+                            uint4 v;
+                            v.x = pack_bf16x2(__uint_as_float(o[8 * j + 0]) * inv, __uint_as_float(o[8 * j + 1]) * inv);
+                            v.y = pack_bf16x2(__uint_as_float(o[8 * j + 2]) * inv, __uint_as_float(o[8 * j + 3]) * inv);
+                            v.z = pack_bf16x2(__uint_as_float(o[8 * j + 4]) * inv, __uint_as_float(o[8 * j + 5]) * inv);
+                            v.w = pack_bf16x2(__uint_as_float(o[8 * j + 6]) * inv, __uint_as_float(o[8 * j + 7]) * inv);
+                            orow[c * 4 + j] = v;
+                        }
                     }
                 }
+                if (row_ok) p.lse[tok * p.num_q_heads + head] = (m_run + log2f(l)) * kLn2;
+            } else {
+                // a key split: store O / l and m + log2 l of this split (the
+                // partial of Eq. 1 over its keys), row r of the tile at float4
+                // column q in position q * 128 + r, so that a warp's stores
+                // and loads are contiguous
+                const int64_t prow = (static_cast<int64_t>(it.pbase + it.split) * 2 + w) * 128;
+                float4 *po = reinterpret_cast<float4 *>(p.ppart_o) + prow * (D / 4) + r;
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
+                    tc::tmem_wait_ld();
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        po[(c * 8 + j) * 128] = make_float4(__uint_as_float(o[4 * j]) * inv, __uint_as_float(o[4 * j + 1]) * inv,
+                                                            __uint_as_float(o[4 * j + 2]) * inv, __uint_as_float(o[4 * j + 3]) * inv);
+                }
+                const float my_lse = m_run + log2f(l);
+                p.ppart_lse[prow + r] = my_lse;
+                // the last split of this tile pair to finish merges, warp by warp
+                __threadfence();
+                __syncwarp();
+                int last = 0;
+                if (lane == 0) last = atomicAdd(p.pcounters + it.cnt * 8 + (warp & 7), 1) == it.ns - 1;
+                last = __shfl_sync(0xffffffffu, last, 0);
+                if (last) {
+                    __threadfence();
+                    auto lse_of = [&](int sp) {
+                        return __ldcg(p.ppart_lse + (static_cast<int64_t>(it.pbase + sp) * 2 + w) * 128 + r);
+                    };
+                    // sums run in split order, whichever split merges, so
+                    // that a run is reproducible bit for bit
+                    float M = -INFINITY;
+                    for (int sp = 0; sp < it.ns; ++sp) M = fmaxf(M, sp == it.split ? my_lse : lse_of(sp));
+                    float L = 0.f;
+                    for (int sp = 0; sp < it.ns; ++sp) L += fast_exp2((sp == it.split ? my_lse : lse_of(sp)) - M);
+                    const float iL = 1.f / L;
+#pragma unroll 1
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
+                        tc::tmem_wait_ld();
+                        float4 acc[8];
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+                        for (int sp = 0; sp < it.ns; ++sp) {
+                            float4 v[8];
+                            float ws;
+                            if (sp == it.split) {
+                                ws = fast_exp2(my_lse - M);
+#pragma unroll
+                                for (int j = 0; j < 8; ++j)
+                                    v[j] = make_float4(__uint_as_float(o[4 * j]) * inv, __uint_as_float(o[4 * j + 1]) * inv,
+                                                       __uint_as_float(o[4 * j + 2]) * inv, __uint_as_float(o[4 * j + 3]) * inv);
+                            } else {
+                                ws = fast_exp2(lse_of(sp) - M);
+                                const float4 *q4 = reinterpret_cast<const float4 *>(p.ppart_o) +
+                                                   (static_cast<int64_t>(it.pbase + sp) * 2 + w) * 128 * (D / 4) + r;
+#pragma unroll
+                                for (int j = 0; j < 8; ++j) v[j] = __ldcg(q4 + (c * 8 + j) * 128);
+                            }
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) {
+                                acc[j].x += ws * v[j].x; acc[j].y += ws * v[j].y;
+                                acc[j].z += ws * v[j].z; acc[j].w += ws * v[j].w;
+                            }
+                        }
+                        if (row_ok) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                uint4 v;
+                                v.x = pack_bf16x2(acc[2 * j].x * iL, acc[2 * j].y * iL);
+                                v.y = pack_bf16x2(acc[2 * j].z * iL, acc[2 * j].w * iL);
+                                v.z = pack_bf16x2(acc[2 * j + 1].x * iL, acc[2 * j + 1].y * iL);
+                                v.w = pack_bf16x2(acc[2 * j + 1].z * iL, acc[2 * j + 1].w * iL);
+                                orow[c * 4 + j] = v;
+                            }
+                        }
+                    }
+                    if (row_ok) p.lse[tok * p.num_q_heads + head] = (M + log2f(L)) * kLn2;
+                    if (lane == 0) p.pcounters[it.cnt * 8 + (warp & 7)] = 0;  // ready for the next run
+                }
             }
-            if (row_ok) p.lse[tok * p.num_q_heads + head] = (m_run + log2f(l)) * kLn2;
             t += it.ntiles;
             tc::fence_before_sync();
             tc::mbar_arrive(ITEMEMPTY(slot));

@@ -262,3 +262,26 @@ def test_decode_four_kv_heads_edges(bs, split):
     st = _step(batch, split=split)
     out, lse = st.results()
     _compare(batch, out, lse)
+
+
+@pytest.mark.parametrize("bs", [16, 64])
+@pytest.mark.parametrize("dim", [64, 128])
+def test_prefill_key_splits(bs, dim):
+    """Few prefill tiles over long cached prefixes: the planner splits their
+    keys across CTAs and the last split merges the partial results. Chunks of
+    one row, ragged chunks and prefixes off block edges, beside decodes."""
+    sh = W.Shape(8, 2, dim, dim, bs, False)
+    ql = [40, 1, 200, 1, 77]
+    ctx = [3040, 5000, 2500, 900, 77 + 1999]
+    ph = [0, 0, 0, 1, 0]
+    rng = np.random.default_rng(31 * bs + dim)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="ksplit")
+    st = _step(batch)
+    units = sum((q + 63) // 64 * 2 for q, p in zip(ql, ph) if p == 0)  # tile pairs x kv heads
+    assert st.plan.info()["prefill_items"] > units, "expected the planner to split prefill keys"
+    out, lse = st.results()
+    _compare(batch, out, lse)
+    for _ in range(2):  # the merge counters are back at zero after a run
+        st.run()
+    out2, lse2 = st.results()
+    assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
