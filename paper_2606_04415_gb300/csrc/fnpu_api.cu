@@ -45,6 +45,13 @@ struct fnpu_plan {
     float *d_ppart_lse = nullptr;
     float *d_ppart_o = nullptr;
     int32_t num_pparts = 0, num_pgroups = 0;
+    // co-location (Sec. 3.4): prefill CTAs on pre_ctas SMs and decode CTAs on
+    // the others, launched together on two library streams forked from and
+    // joined back into the caller's stream
+    bool coloc = false;
+    int32_t pre_ctas = 0;
+    cudaStream_t s_pre = nullptr, s_dec = nullptr;
+    cudaEvent_t e_fork = nullptr, e_pre = nullptr, e_dec = nullptr;
 };
 
 namespace fnpu {
@@ -60,6 +67,43 @@ int cuda_fail(cudaError_t e, const char *where) {
 namespace {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+void destroy_sync_objects(fnpu_plan *pl) {
+    if (pl->s_pre) cudaStreamDestroy(pl->s_pre);
+    if (pl->s_dec) cudaStreamDestroy(pl->s_dec);
+    if (pl->e_fork) cudaEventDestroy(pl->e_fork);
+    if (pl->e_pre) cudaEventDestroy(pl->e_pre);
+    if (pl->e_dec) cudaEventDestroy(pl->e_dec);
+    pl->s_pre = pl->s_dec = nullptr;
+    pl->e_fork = pl->e_pre = pl->e_dec = nullptr;
+}
+
+// Modelled rates of the two phases: a prefill CTA finishes one 64-key tile of
+// both Q tiles (d = 128) in about 0.93 us; a decode SM streams about 60 GB/s of
+// KV cache and the whole device about 4 TB/s.
+constexpr double kTileSec = 0.93e-6;
+constexpr double kDecodeSmBps = 60e9;
+constexpr double kDecodeAllBps = 4.0e12;
+
+// SMs that start on decode while the others run prefill: prefill on sms - k
+// SMs lasts Tp; decode streams at min(all, k * per SM) meanwhile, and what is
+// left runs on every SM once the prefill CTAs have finished. The k with the
+// shortest modelled step wins.
+int32_t choose_decode_sms(int64_t pre_tiles, int64_t dec_bytes, int32_t sms) {
+    int32_t best_k = 1;
+    double best_t = -1.0;
+    for (int32_t k = 1; k <= sms / 2; ++k) {
+        const double tp = static_cast<double>(pre_tiles) * kTileSec / (sms - k);
+        const double rate = std::min(kDecodeAllBps, k * kDecodeSmBps);
+        const double left = std::max(0.0, static_cast<double>(dec_bytes) - tp * rate);
+        const double t = tp + left / kDecodeAllBps;
+        if (best_t < 0 || t < best_t) {
+            best_t = t;
+            best_k = k;
+        }
+    }
+    return best_k;
+}
 
 // Two packed Q tiles of one kv head (the tcgen05 prefill unit) before its key
 // range is split.
@@ -349,9 +393,27 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         }
         qs += query_len[s];
     }
+    // co-location: the decode CTAs take a share of the SMs while the prefill
+    // CTAs hold the rest
+    pl->coloc = pl->use_tc && pl->use_dt && !tc_units.empty() && !ditems.empty() &&
+                !(o.flags & FNPU_PLAN_SEPARATE_LAUNCHES);
+    pl->pre_ctas = sms;
+    if (pl->coloc) {
+        int64_t dec_bytes = 0;
+        for (const DecodeItem &it : ditems)
+            dec_bytes += static_cast<int64_t>(it.key_end - it.key_begin) * desc->num_kv_heads *
+                         (desc->head_dim_qk + desc->head_dim_v) * 2;
+        int64_t pre_tiles = 0;
+        for (const TcUnit &u : tc_units) pre_tiles += u.ntiles + kTcItemCost;
+        pre_tiles = pre_tiles * (desc->head_dim_qk + desc->head_dim_v) / 256;  // in d = 128 tiles
+        const int32_t k = o.decode_share_pct > 0
+                              ? std::min(sms - 1, std::max(1, (sms * o.decode_share_pct + 50) / 100))
+                              : choose_decode_sms(pre_tiles, dec_bytes, sms);
+        pl->pre_ctas = sms - k;
+    }
     int32_t pparts = 0, pgroups = 0;
     if (!tc_units.empty()) {
-        const std::vector<int32_t> ns = choose_prefill_splits(tc_units, sms);
+        const std::vector<int32_t> ns = choose_prefill_splits(tc_units, pl->pre_ctas);
         for (size_t u = 0; u < tc_units.size(); ++u) {
             const TcUnit &t = tc_units[u];
             const int32_t n = ns[u];
@@ -386,6 +448,20 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->num_parts = parts;
     pl->num_pparts = pparts;
     pl->num_pgroups = pgroups;
+    if (pl->coloc) {
+        int lo = 0, hi = 0;
+        if (cudaDeviceGetStreamPriorityRange(&lo, &hi) != cudaSuccess ||
+            cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess ||
+            cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pl->e_fork, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pl->e_pre, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pl->e_dec, cudaEventDisableTiming) != cudaSuccess) {
+            cudaGetLastError();
+            destroy_sync_objects(pl);
+            delete pl;
+            return FNPU_ECUDA;
+        }
+    }
 
     // workspace: metadata (uploaded) then scratch (never read before written)
     size_t off = 0;
@@ -406,12 +482,14 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
 
     if (cudaMalloc(&pl->d_ws, pl->ws_bytes) != cudaSuccess) {
         cudaGetLastError();
+        destroy_sync_objects(pl);
         delete pl;
         return FNPU_ENOMEM;
     }
     if (cudaMallocHost(&pl->h_stage, meta_bytes) != cudaSuccess) {
         cudaGetLastError();
         cudaFree(pl->d_ws);
+        destroy_sync_objects(pl);
         delete pl;
         return FNPU_ENOMEM;
     }
@@ -442,6 +520,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         cudaGetLastError();
         cudaFreeHost(pl->h_stage);
         cudaFree(pl->d_ws);
+        destroy_sync_objects(pl);
         delete pl;
         return FNPU_ECUDA;
     }
@@ -494,10 +573,29 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
 
+    if (pl->coloc) {
+        // both phases at once: pre_ctas persistent prefill CTAs (one per SM,
+        // the tensor pipe; a decode CTA does not fit beside one) and decode
+        // CTAs on the other SMs (HBM). The prefill stream has the higher
+        // priority, so its CTAs are placed first; decode CTAs beyond the
+        // free SMs start on the SMs that the prefill leaves as its queue
+        // runs dry.
+        cudaStream_t s = static_cast<cudaStream_t>(stream);
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
+        int rc = launch_prefill_tc(p, pl->s_pre, pl->pre_ctas);
+        if (rc == FNPU_OK) rc = launch_decode_tma(p, pl->s_dec, 3 * pl->num_sms);
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_pre, 0));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
+        return rc;
+    }
     int rc = pl->use_dt ? launch_decode_tma(p, stream, 3 * pl->num_sms)
                         : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
-    return pl->use_tc ? launch_prefill_tc(p, stream) : launch_prefill_mma(p, stream);
+    return pl->use_tc ? launch_prefill_tc(p, stream, pl->num_sms) : launch_prefill_mma(p, stream);
 }
 
 int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
@@ -523,6 +621,7 @@ int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
 void fnpu_plan_destroy(fnpu_plan *pl) {
     if (!pl) return;
     cudaDeviceSynchronize();
+    destroy_sync_objects(pl);
     if (pl->h_stage) cudaFreeHost(pl->h_stage);
     if (pl->d_ws) cudaFree(pl->d_ws);
     delete pl;

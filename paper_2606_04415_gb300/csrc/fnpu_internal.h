@@ -91,7 +91,7 @@ int launch_decode_mma(const AttnParams &p, void *stream);
 int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas);
 bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_prefill_mma(const AttnParams &p, void *stream);
-int launch_prefill_tc(const AttnParams &p, void *stream);
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
 int prefill_tc_rows_per_item(int group);
 

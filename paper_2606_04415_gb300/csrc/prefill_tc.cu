@@ -646,7 +646,7 @@ bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, in
 }
 
 template <int D>
-int launch_tc(const AttnParams &p, cudaStream_t st) {
+int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas) {
     using Cfg = TcCfg<D>;
     TcMaps maps;
     if (!encode_cache_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
@@ -655,10 +655,9 @@ int launch_tc(const AttnParams &p, cudaStream_t st) {
         return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
     FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmemBytes));
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int grid = p.num_pitems < sms ? p.num_pitems : sms;
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                       cudaSharedmemCarveoutMaxShared));
+    const int grid = p.num_pitems < max_ctas ? p.num_pitems : max_ctas;
     prefill_tc_kernel<D><<<grid, kThreads, Cfg::kSmemBytes, st>>>(p, maps);
     FNPU_CUDA_TRY(cudaGetLastError());
     return FNPU_OK;
@@ -674,12 +673,12 @@ bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group) {
 // positions per work item: two Q tiles of floor(128 / G) positions each
 int prefill_tc_rows_per_item(int group) { return 2 * (kRows / group); }
 
-int launch_prefill_tc(const AttnParams &p, void *stream) {
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas) {
     if (p.num_pitems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     switch (p.head_dim_qk) {
-        case 64: return launch_tc<64>(p, st);
-        case 128: return launch_tc<128>(p, st);
+        case 64: return launch_tc<64>(p, st, max_ctas);
+        case 128: return launch_tc<128>(p, st, max_ctas);
         default: return FNPU_EUNSUPPORTED;
     }
 }

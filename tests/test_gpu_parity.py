@@ -285,3 +285,22 @@ def test_prefill_key_splits(bs, dim):
         st.run()
     out2, lse2 = st.results()
     assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
+
+
+SEPARATE = 1  # FNPU_PLAN_SEPARATE_LAUNCHES
+
+
+@pytest.mark.parametrize("share", [0, 2, 50])
+def test_colocated_launch_matches_separate_launches(share):
+    """Prefill and decode launched together on split SMs (any decode share)
+    give the results of the two phases launched one after the other."""
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(77)
+    ql = [300, 1, 1, 129, 1] + [1] * 12
+    ctx = [300 + 2000, 700, 1500, 129 + 40, 33] + list(rng.integers(20, 3000, size=12))
+    ph = [0, 1, 1, 0, 1] + [1] * 12
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="coloc_small")
+    a_out, a_lse = _step(batch, share=share).results()
+    b_out, b_lse = _step(batch, flags=SEPARATE).results()
+    _compare(batch, a_out, a_lse)
+    assert np.abs(a_out - b_out).max() <= O_TOL and np.abs(a_lse - b_lse).max() <= LSE_TOL
