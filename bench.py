@@ -41,6 +41,16 @@ METRIC = "mixed PD attention query tokens/s at 1 GB300; % of max(FLOP,HBM) roofl
 UNIT = "query tokens/s"
 L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 
+# DRAM bytes (read + write) of one attention call, from ncu captures of the
+# current kernels (dram__bytes_read.sum + dram__bytes_write.sum; for the
+# co-located step the sum over its prefill and decode launches); the
+# summaries with the commands are under profiles/. Set to None for a
+# workload whose kernels change until they are captured again.
+NCU_TRAFFIC = {
+    "qwen_coloc": 491.8e6,   # prefill_tc 33.4 MB + decode_tma 458.3 MB
+    "qwen_decode": 326.0e6,  # decode_tma 315.3 MB read + 10.7 MB write
+}
+
 
 def _flush_l2(wbuf, rbuf):
     """Evict L2 between timed steps: write a buffer larger than L2, then read
@@ -311,7 +321,7 @@ def run_fnpu(args):
     else:
         roof = {"bound": "hbm", "achieved": B_attn / t_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = args.traffic
+    roof["traffic"] = args.traffic if args.traffic is not None else NCU_TRAFFIC.get(args.workload)
     roof["peak_source"] = peaks["source"] + " burst"
     step_roof = max(F / (peaks["bf16_tflops"] * 1e12), work["bytes"] / (peaks["hbm_gbs"] * 1e9))
     step_roof_sus = max(F / (peaks["bf16_tflops_sustained"] * 1e12), work["bytes"] / (peaks["hbm_gbs"] * 1e9))
