@@ -28,7 +28,10 @@ struct fnpu_plan {
     int32_t num_sms = 0;
     int32_t flags = 0;
     bool use_tc = false;
-    bool use_dt = false;  // decode on the TMA-fed persistent kernel (items cover all kv heads)
+    bool use_dt = false;
+    bool use_mla = false;  // latent attention: one work list for both phases
+    int32_t num_mitems = 0;
+    fnpu::MlaItem *d_mitems = nullptr;  // decode on the TMA-fed persistent kernel (items cover all kv heads)
     int32_t num_ditems = 0, num_pitems = 0, num_groups = 0, num_parts = 0;
     void *d_ws = nullptr;
     size_t ws_bytes = 0;
@@ -191,9 +194,12 @@ bool shape_ok(const fnpu_attn_desc *d, int *status) {
     return true;
 }
 
-// Kernels exist for split K/V with d in {64, 128} (decode needs G <= 8).
+// Kernels exist for split K/V with d in {64, 128} (decode needs G <= 8) and
+// for the latent layout with d_qk = 576, d_v = 512 and a multiple of 64 heads.
 int kernel_support(const fnpu_attn_desc *d, bool has_decode) {
-    if (d->v_in_k_latent) return FNPU_EUNSUPPORTED;
+    if (d->v_in_k_latent)
+        return mla_supported(d->head_dim_qk, d->head_dim_v, d->num_q_heads, d->num_kv_heads) ? FNPU_OK
+                                                                                               : FNPU_EUNSUPPORTED;
     if (d->head_dim_qk != d->head_dim_v) return FNPU_EUNSUPPORTED;
     if (d->head_dim_qk != 64 && d->head_dim_qk != 128) return FNPU_EUNSUPPORTED;
     if (has_decode && d->num_q_heads / d->num_kv_heads > 8) return FNPU_EUNSUPPORTED;
@@ -315,9 +321,10 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->bt_width = width;
     pl->num_sms = sms;
     pl->flags = o.flags;
-    pl->use_dt = decode_tma_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_kv_heads,
-                                      desc->num_q_heads / desc->num_kv_heads, bs);
-    pl->use_tc = !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
+    pl->use_mla = desc->v_in_k_latent != 0;
+    pl->use_dt = !pl->use_mla && decode_tma_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_kv_heads,
+                                                      desc->num_q_heads / desc->num_kv_heads, bs);
+    pl->use_tc = !pl->use_mla && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
                  prefill_tc_supported(desc->head_dim_qk, desc->head_dim_v, bs,
                                       desc->num_q_heads / desc->num_kv_heads);
 
@@ -342,11 +349,46 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         split = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(sk, pl->use_dt ? 128 : 256), 4096));
     }
 
+    // latent attention: every query row (prefill or decode) is 64-head blocks
+    // over its visible keys, split into pieces of at most mla_split keys so
+    // that about three CTAs per SM share the work; longest first
+    std::vector<MlaItem> mitems;
+    int32_t mla_split = 0;
+    if (pl->use_mla) {
+        int64_t rows_keys = 0;
+        for (int32_t s = 0; s < num_seqs; ++s) {
+            const int64_t q = query_len[s], p0 = context_len[s] - query_len[s];
+            rows_keys += q * p0 + q * (q + 1) / 2;
+        }
+        rows_keys *= desc->num_q_heads / mla_heads_per_item();
+        const int64_t target = 3LL * sms;
+        int64_t sk = (rows_keys + target - 1) / target;
+        sk = std::max<int64_t>((sk + 255) / 256 * 256, 1024);
+        mla_split = static_cast<int32_t>(std::min<int64_t>(sk, 1 << 20));
+    }
+
     int32_t qs = 0, parts = 0, groups = 0;
     for (int32_t s = 0; s < num_seqs; ++s) {
         seqs[s] = SeqInfo{qs, query_len[s], context_len[s], s};
         const int32_t q = query_len[s], c = context_len[s];
-        if (phase[s] == 1 && pl->use_dt) {
+        if (pl->use_mla) {
+            const int32_t nhb = desc->num_q_heads / mla_heads_per_item();
+            for (int32_t i = 0; i < q; ++i) {
+                const int32_t keys = c - q + i + 1;
+                const int32_t ns = (keys + mla_split - 1) / mla_split;
+                const int32_t sk = (keys + ns - 1) / ns;  // even pieces
+                for (int32_t hb = 0; hb < nhb; ++hb) {
+                    const int32_t base = ns > 1 ? parts : 0, grp = ns > 1 ? groups : 0;
+                    if (ns > 1) {
+                        parts += ns;
+                        groups += 1;
+                    }
+                    for (int32_t sp = 0; sp < ns; ++sp)
+                        mitems.push_back(MlaItem{s, i, hb, sp * sk, std::min(keys, (sp + 1) * sk), sp, ns, base, grp,
+                                                 0, 0, 0});
+                }
+            }
+        } else if (phase[s] == 1 && pl->use_dt) {
             // items over all kv heads; one merge counter per (sequence, kv head)
             const int32_t sk = std::max(split, (c + 255 * 64) / (256 * 64) * 64);
             const int32_t ns = (c + sk - 1) / sk;
@@ -442,6 +484,10 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         return (a.key_end - a.key_begin) > (b.key_end - b.key_begin);
     });
 
+    std::stable_sort(mitems.begin(), mitems.end(), [](const MlaItem &a, const MlaItem &b) {
+        return (a.key_end - a.key_begin) > (b.key_end - b.key_begin);
+    });
+    pl->num_mitems = static_cast<int32_t>(mitems.size());
     pl->num_ditems = static_cast<int32_t>(ditems.size());
     pl->num_pitems = static_cast<int32_t>(pordered.size());
     pl->num_groups = groups;
@@ -468,12 +514,14 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_seqs = off; off = align_up(off + sizeof(SeqInfo) * std::max(num_seqs, 1), 256);
     const size_t o_bt = off; off = align_up(off + sizeof(int32_t) * static_cast<size_t>(std::max(num_seqs, 1)) * width, 256);
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
+    const size_t o_mi = off; off = align_up(off + sizeof(MlaItem) * std::max<size_t>(mitems.size(), 1), 256);
     const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
     const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
     const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
     const size_t meta_bytes = off;
-    const int32_t part_rows = pl->use_dt ? desc->num_q_heads : G;  // query heads per partial
+    // query heads per partial
+    const int32_t part_rows = pl->use_mla ? mla_heads_per_item() : (pl->use_dt ? desc->num_q_heads : G);
     const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows, 256);
     const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows * desc->head_dim_v, 256);
     const size_t o_pplse = off; off = align_up(off + sizeof(float) * 256 * static_cast<size_t>(std::max(pparts, 1)), 256);
@@ -501,12 +549,14 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                block_table + static_cast<int64_t>(s) * block_table_stride,
                sizeof(int32_t) * static_cast<size_t>((context_len[s] + bs - 1) / bs));
     if (!ditems.empty()) memcpy(h + o_di, ditems.data(), sizeof(DecodeItem) * ditems.size());
+    if (!mitems.empty()) memcpy(h + o_mi, mitems.data(), sizeof(MlaItem) * mitems.size());
     if (!pordered.empty()) memcpy(h + o_pi, pordered.data(), sizeof(PrefillItem) * pordered.size());
 
     uint8_t *d = static_cast<uint8_t *>(pl->d_ws);
     pl->d_seqs = reinterpret_cast<SeqInfo *>(d + o_seqs);
     pl->d_bt = reinterpret_cast<int32_t *>(d + o_bt);
     pl->d_ditems = reinterpret_cast<DecodeItem *>(d + o_di);
+    pl->d_mitems = reinterpret_cast<MlaItem *>(d + o_mi);
     pl->d_pitems = reinterpret_cast<PrefillItem *>(d + o_pi);
     pl->d_counters = reinterpret_cast<int32_t *>(d + o_cnt);
     pl->d_err = reinterpret_cast<int32_t *>(d + o_err);
@@ -561,6 +611,8 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.v_slot_stride = latent ? d.head_dim_qk : static_cast<int64_t>(d.num_kv_heads) * d.head_dim_v;
     p.scale_log2 = pl->scale * 1.4426950408889634f;
     p.ditems = pl->d_ditems;
+    p.mitems = pl->d_mitems;
+    p.num_mitems = pl->num_mitems;
     p.num_ditems = pl->num_ditems;
     p.part_o = pl->d_part_o;
     p.part_lse = pl->d_part_lse;
@@ -573,6 +625,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
 
+    if (pl->use_mla) return launch_mla(p, stream);
     if (pl->coloc) {
         // both phases at once: pre_ctas persistent prefill CTAs (one per SM,
         // the tensor pipe; a decode CTA does not fit beside one) and decode
@@ -630,9 +683,10 @@ void fnpu_plan_destroy(fnpu_plan *pl) {
 int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_items,
                    int32_t *launches_per_run, int64_t *workspace_bytes) {
     if (!pl) return FNPU_EINVAL;
-    if (prefill_items) *prefill_items = pl->num_pitems;
+    // latent attention has one work list for both phases, reported as prefill items
+    if (prefill_items) *prefill_items = pl->num_pitems + pl->num_mitems;
     if (decode_items) *decode_items = pl->num_ditems;
-    if (launches_per_run) *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0);
+    if (launches_per_run) *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0);
     if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_bytes);
     return FNPU_OK;
 }

@@ -34,6 +34,17 @@ struct PrefillItem {
 };
 static_assert(sizeof(PrefillItem) == 48, "PrefillItem layout");
 
+// One latent-attention (MLA) work item: query heads [64 hb, 64 hb + 64) of
+// query row `row` of sequence `seq` (a prefill or a decode row alike) over
+// keys [key_begin, key_end); splits of one (token, head block) share `group`
+// and write partials to scratch rows part_base + split.
+struct MlaItem {
+    int32_t seq, row, hb, key_begin;
+    int32_t key_end, split, num_splits, part_base;
+    int32_t group, pad0, pad1, pad2;
+};
+static_assert(sizeof(MlaItem) == 48, "MlaItem layout");
+
 // Per-sequence metadata on the device.
 struct SeqInfo {
     int32_t q_start;  // first query token of the sequence in q/out/lse
@@ -70,6 +81,9 @@ struct AttnParams {
     float *ppart_o;         // fp32 split-prefill partials, per partial: [2 tiles][dv / 4][128 rows] float4
     float *ppart_lse;       // fp32 [num_pparts, 2, 128] (log2 domain)
     int32_t *pcounters;     // [num_pgroups, 8] one per softmax warp, zero between runs
+    // latent attention (MLA): one work list for both phases
+    const MlaItem *mitems;
+    int32_t num_mitems;
     int32_t *err;           // device error flag of the plan
     int32_t *sched;         // persistent work queues: [0..1] prefill, [2..3] decode (next item, finished CTAs)
 };
@@ -91,6 +105,9 @@ int launch_decode_mma(const AttnParams &p, void *stream);
 int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas);
 bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_prefill_mma(const AttnParams &p, void *stream);
+int launch_mla(const AttnParams &p, void *stream);
+bool mla_supported(int d_qk, int d_v, int hq, int hkv);
+int mla_heads_per_item();
 int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
 int prefill_tc_rows_per_item(int group);

@@ -96,6 +96,11 @@ def test_plan_reports_unsupported_head_dims():
     bt = np.zeros((1, 4), np.int32)
     desc = fnpu.make_desc(**dict(QWEN, head_dim_qk=96, head_dim_v=96))
     assert _plan_rc(desc, [1], [5], [1], bt) == fnpu.FNPU_EUNSUPPORTED
+    # latent layout: 576 / 512 with a multiple of 64 query heads only
+    lat = fnpu.make_desc(100, 1, 576, 512, 64, 8, latent=True)
+    assert _plan_rc(lat, [1], [5], [1], bt) == fnpu.FNPU_EUNSUPPORTED
+    lat = fnpu.make_desc(128, 1, 320, 256, 64, 8, latent=True)
+    assert _plan_rc(lat, [1], [5], [1], bt) == fnpu.FNPU_EUNSUPPORTED
 
 
 def test_append_and_run_reject_null_pointers():

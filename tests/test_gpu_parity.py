@@ -304,3 +304,43 @@ def test_colocated_launch_matches_separate_launches(share):
     b_out, b_lse = _step(batch, flags=SEPARATE).results()
     _compare(batch, a_out, a_lse)
     assert np.abs(a_out - b_out).max() <= O_TOL and np.abs(a_lse - b_lse).max() <= LSE_TOL
+
+
+@pytest.mark.parametrize("bs", [16, 64])
+def test_mla_small_mixed_batch_all_rows(bs):
+    """Absorbed MLA (128 heads on one 576-wide latent, V = its first 512
+    columns): prefill chunks with and without prefix, decodes long enough to
+    be split and merged, ragged lengths; every row against the oracle. The
+    latent KV append is bit-exact."""
+    sh = W.Shape(128, 1, 576, 512, bs, True)
+    ql = [7, 1, 1, 33, 1, 1]
+    ctx = [7, 2500, 1, 33 + 450, 777, 3100]
+    ph = [0, 1, 1, 0, 1, 1]
+    rng = np.random.default_rng(500 + bs)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_small")
+    st = _step(batch)
+    kc, _ = st.cache_bits()
+    assert np.array_equal(kc, oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping))
+    out, lse = st.results()
+    _compare(batch, out, lse)
+    st.run()  # merge counters back at zero: a second run is identical
+    out2, lse2 = st.results()
+    assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
+
+
+def test_mla_coloc_full_size_sampled_rows():
+    """The DeepSeek-R1-shaped co-located step at full size (1024-token
+    prefill + 256 decodes up to 16K keys); the oracle recomputes a sample of
+    decode rows and prefill rows."""
+    batch = W.make_batch("mla_coloc", seed=0)
+    st = _step(batch)
+    out, lse = st.results()
+    rng = np.random.default_rng(1)
+    qs = batch.query_start
+    dec = [int(qs[s]) for s in np.flatnonzero(batch.phase == 1)]
+    pre = [s for s in range(batch.num_seqs) if batch.phase[s] == 0]
+    toks = sorted(rng.choice(dec, size=12, replace=False).tolist())
+    for s in pre:
+        q = int(batch.query_len[s])
+        toks += [int(qs[s]) + r for r in sorted({0, 1, 63, 64, q - 1, int(rng.integers(0, q))})]
+    _compare(batch, out, lse, tokens=np.asarray(sorted(set(toks)), np.int64))
