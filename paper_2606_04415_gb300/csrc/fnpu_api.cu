@@ -81,10 +81,10 @@ void destroy_sync_objects(fnpu_plan *pl) {
     pl->e_fork = pl->e_pre = pl->e_dec = nullptr;
 }
 
-// Modelled rates of the two phases: a prefill CTA finishes one 64-key tile of
-// both Q tiles (d = 128) in about 0.93 us; a decode SM streams about 60 GB/s of
-// KV cache and the whole device about 4 TB/s.
-constexpr double kTileSec = 0.93e-6;
+// Modelled rates of the two phases: a prefill CTA finishes one 128-key tile
+// of both Q tiles (d = 128) in about 1.6 us; a decode SM streams about 60 GB/s
+// of KV cache and the whole device about 4 TB/s.
+constexpr double kTileSec = 1.6e-6;
 constexpr double kDecodeSmBps = 60e9;
 constexpr double kDecodeAllBps = 4.0e12;
 
@@ -116,11 +116,11 @@ struct TcUnit {
     int32_t max_start;  // last tile a split may start at: every row must see a key of every split
 };
 
-// Cost model of a prefill work item in units of one 64-key tile of both Q
+// Cost model of a prefill work item in units of one 128-key tile of both Q
 // tiles: switching items (loading Q, draining the pipeline, the epilogue) and,
 // for a split item, writing its partial result and the merge.
 constexpr int64_t kTcItemCost = 2;
-constexpr int64_t kTcMergeCost = 3;
+constexpr int64_t kTcMergeCost = 4;
 
 // First tile of split j of n over ntiles tiles (split n is the end).
 int32_t split_bound(int32_t ntiles, int32_t n, int32_t j) {
@@ -153,12 +153,13 @@ std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int
     }
     std::vector<int64_t> caps = {maxc};
     for (int k = 2; k <= 8; ++k) caps.push_back((maxc + k - 1) / k);
+    // (cap below: pieces shorter than 4 tiles cost more than they balance)
     for (int j = 1; j <= 8; ++j) caps.push_back((total + static_cast<int64_t>(sms) * j - 1) / (static_cast<int64_t>(sms) * j));
     std::vector<int32_t> best(units.size(), 1), ns(units.size(), 1);
     int64_t best_span = -1;
     std::vector<int64_t> costs;
     for (int64_t cap : caps) {
-        if (cap < 8) continue;  // pieces shorter than this cost more than they balance
+        if (cap < 4) continue;
         costs.clear();
         for (size_t i = 0; i < units.size(); ++i) {
             const TcUnit &u = units[i];
@@ -415,12 +416,12 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
             // tcgen05 tiles: two Q tiles of P positions x G heads of one kv
             // head; their key splits are chosen once all tiles are known
             const int32_t prefix = c - q;
-            const int32_t P2 = prefill_tc_rows_per_item(G);
+            const int32_t P2 = prefill_tc_rows_per_item(G), KT = prefill_tc_keys_per_tile();
             for (int32_t r0 = 0; r0 < q; r0 += P2) {
                 const int32_t rows = std::min(P2, q - r0);
-                const int32_t ntiles = (prefix + r0 + rows + 63) / 64;
+                const int32_t ntiles = (prefix + r0 + rows + KT - 1) / KT;
                 for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh)
-                    tc_units.push_back(TcUnit{s, kvh, r0, rows, ntiles, (prefix + r0) / 64});
+                    tc_units.push_back(TcUnit{s, kvh, r0, rows, ntiles, (prefix + r0) / KT});
             }
         } else {
             const int32_t prefix = c - q;

@@ -111,5 +111,6 @@ int mla_heads_per_item();
 int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
 int prefill_tc_rows_per_item(int group);
+int prefill_tc_keys_per_tile();
 
 }  // namespace fnpu

@@ -10,31 +10,33 @@
 // busy for G = 7). A 3-D TMA box (64 columns x G heads x P positions) writes
 // exactly this row order. A work item is two consecutive Q tiles of one kv
 // head (2P positions) that consume the same K/V tiles, which halves the
-// L2-to-SM traffic per FLOP (one Q tile per K/V tile would need about
-// 50 B/clk per SM at the tensor rate).
+// L2-to-SM traffic per FLOP.
+//
+// Key tiles are 128 keys wide: an S = Q K^T product is then M = N = 128 and
+// runs at the full tensor rate (a 64-wide one, with both operands in shared
+// memory, is bound by shared-memory bandwidth: 48 instead of 32 cycles).
 //
 // One persistent CTA per SM (384 threads) takes items, longest first, from an
 // atomic queue (the last CTA to finish resets it for the next run):
 //   warps 0-3, 4-7  softmax warpgroups for Q tile 0 and tile 1, one MMA row
-//                   per thread: online softmax on the S row read from TMEM,
-//                   P (bf16) written over S, lazy rescale of the O row,
+//                   per thread: the 128 scores of the row from TMEM into
+//                   registers, online softmax, P (bf16) written back over the
+//                   first 64 columns of S, lazy rescale of the O row,
 //                   epilogue;
 //   warp 8          scheduler and K producer: the item's two Q tiles, then the
-//                   64-key K tiles gathered block by block through the block
-//                   table (one 4-D box per block and 64-column half);
-//   warp 9          V producer for the same tiles; zeroes V rows past the
-//                   context before the last PV of an item. Each TMA issue
-//                   costs on the order of a hundred cycles per issuing warp,
-//                   so K and V are issued from separate warps;
-//   warps 10, 11    issue the MMAs (warp-uniform, one elected lane); warp 10
-//                   issues S_w(j+1) = Q_w K(j+1)^T as soon as warpgroup w has
-//                   copied S_w(j) into registers, warp 11 issues
-//                   O_w += P_w(j) V(j) as soon as P_w(j) is written. The MMA
-//                   queue is short, so one warp's barrier waits would leave the
-//                   tensor core idle; two issuers keep it fed.
-// TMEM (512 columns): S0 at 0, S1 at 64 (fp32); P0 at 128/160 and P1 at
-// 192/224 (bf16, double-buffered); O0 at 256, O1 at 384. Because P has its
-// own buffers, no S MMA ever waits for a PV to drain.
+//                   128-key K tiles gathered block by block through the block
+//                   table (one 4-D box per block and 64-column half) into a
+//                   3-stage ring;
+//   warp 9          V producer (2-stage ring); zeroes V rows past the context
+//                   before the last PV of an item;
+//   warp 10         issues every MMA, in the order PV_0(j), S_0(j+1), PV_1(j),
+//                   S_1(j+1): the tensor pipe completes a thread's MMAs in
+//                   issue order, so S_w(j+1) overwrites P_w(j) only after
+//                   PV_w(j) has read it, and when S_w(j) is complete so is
+//                   PV_w(j-1) -- the softmax may rescale O_w at that point
+//                   without a further wait.
+// TMEM (512 columns): S0 at 0, S1 at 128 (fp32, P over their first 64
+// columns); O0 at 256, O1 at 384.
 // Every mbarrier wait is bounded; a timeout raises the plan's error flag and
 // the CTA drains its tensor-core work, frees its tensor memory and exits.
 #include <math.h>
@@ -49,27 +51,32 @@ namespace {
 
 constexpr int kThreads = 384;
 constexpr int kRows = 128;
-constexpr int kKeys = 64;
-constexpr int kStages = 4;
+constexpr int kKeys = 128;   // keys per tile
+constexpr int kKStages = 3;  // K ring
+constexpr int kVStages = 2;  // V ring
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p <= 2^8 before a rescale
+// Register split (setmaxnreg): the softmax warpgroups hold a 128-score row
+// each; the producer and MMA warpgroup needs few.
+constexpr uint32_t kRegsSoftmax = 208;
+constexpr uint32_t kRegsHelper = 88;
+static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsHelper <= 65536 / kThreads / 8 * 8 * kThreads, "register split");
 
-__host__ __device__ constexpr uint32_t col_s(int w) { return 64u * w; }
-__host__ __device__ constexpr uint32_t col_p(int w, int b) { return 128u + 64u * w + 32u * b; }
+__host__ __device__ constexpr uint32_t col_s(int w) { return 128u * w; }
 __host__ __device__ constexpr uint32_t col_o(int w) { return 256u + 128u * w; }
 
 template <int D>
 struct TcCfg {
     static constexpr int kTileBytes = kKeys * D * 2;  // one K or V tile
-    static constexpr int kStageBytes = 2 * kTileBytes;
     static constexpr int kHalf = kKeys * 128;         // one 64-column half of a K/V tile
     static constexpr int kQHalf = kRows * 128;        // one 64-column half of a Q tile
     static constexpr int kQBytes = kRows * D * 2;     // one Q tile
-    static constexpr int kQOff = kStages * kStageBytes;
+    static constexpr int kVOff = kKStages * kTileBytes;
+    static constexpr int kQOff = kVOff + kVStages * kTileBytes;
     static constexpr int kBarOff = kQOff + 2 * kQBytes;
-    // kfull[S] vfull[S] kempty[S] vempty[S] sfull[2] sfree[2] pfull[2][2] pvdone[2][2]
-    // qfull qempty vzero itemfull[2] itemempty[2] drain[2]
-    static constexpr int kNumBars = 4 * kStages + 12 + 9;
+    // kfull[3] kempty[3] vfull[2] vempty[2] sfull[2] pfull[2] odone[2] ofree[2]
+    // qfull qempty vzero itemfull[2] itemempty[2] drain
+    static constexpr int kNumBars = 2 * kKStages + 2 * kVStages + 8 + 3 + 4 + 1;
     static constexpr int kSmemUsed = kBarOff + 8 * kNumBars + 32;
     // at least 116 KB so that no two CTAs share an SM (each holds all 512 TMEM columns)
     static constexpr int kSmemBytes = kSmemUsed > 116 * 1024 ? kSmemUsed : 116 * 1024;
@@ -95,7 +102,7 @@ __device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
     g.rows = it.rows;
     g.prefix = si.ctx_len - si.q_len;
     g.ctx = si.ctx_len;
-    g.kt0 = it.kt_begin;              // 64-key tiles [kt_begin, kt_end) of keys 0 .. last position
+    g.kt0 = it.kt_begin;              // 128-key tiles [kt_begin, kt_end) of keys 0 .. last position
     g.ntiles = it.kt_end - it.kt_begin;
     g.q_start = si.q_start;
     g.bt_row = si.bt_row;
@@ -115,18 +122,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t s_base = smem_u32(smem);
     const uint32_t s_bars = s_base + Cfg::kBarOff;
     auto KFULL = [&](int s) { return s_bars + 8 * s; };
-    auto VFULL = [&](int s) { return s_bars + 8 * (kStages + s); };
-    auto KEMPTY = [&](int s) { return s_bars + 8 * (2 * kStages + s); };
-    auto VEMPTY = [&](int s) { return s_bars + 8 * (3 * kStages + s); };
-    const uint32_t b0 = s_bars + 8 * (4 * kStages);
+    auto KEMPTY = [&](int s) { return s_bars + 8 * (kKStages + s); };
+    auto VFULL = [&](int s) { return s_bars + 8 * (2 * kKStages + s); };
+    auto VEMPTY = [&](int s) { return s_bars + 8 * (2 * kKStages + kVStages + s); };
+    const uint32_t b0 = s_bars + 8 * (2 * kKStages + 2 * kVStages);
     auto SFULL = [&](int w) { return b0 + 8 * w; };
-    auto SFREE = [&](int w) { return b0 + 16 + 8 * w; };
-    auto PFULL = [&](int w, int b) { return b0 + 32 + 8 * (2 * w + b); };
-    auto PVDONE = [&](int w, int b) { return b0 + 64 + 8 * (2 * w + b); };
-    const uint32_t QFULL = b0 + 96, QEMPTY = b0 + 104, VZERO = b0 + 112;
-    auto ITEMFULL = [&](int k) { return b0 + 120 + 8 * k; };
-    auto ITEMEMPTY = [&](int k) { return b0 + 136 + 8 * k; };
-    auto DRAIN = [&](int i) { return b0 + 152 + 8 * i; };
+    auto PFULL = [&](int w) { return b0 + 16 + 8 * w; };
+    auto ODONE = [&](int w) { return b0 + 32 + 8 * w; };
+    auto OFREE = [&](int w) { return b0 + 48 + 8 * w; };
+    const uint32_t QFULL = b0 + 64, QEMPTY = b0 + 72, VZERO = b0 + 80;
+    auto ITEMFULL = [&](int k) { return b0 + 88 + 8 * k; };
+    auto ITEMEMPTY = [&](int k) { return b0 + 104 + 8 * k; };
+    const uint32_t DRAIN = b0 + 120;
     uint8_t *misc = smem + Cfg::kBarOff + 8 * Cfg::kNumBars;
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(misc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 4);
@@ -141,27 +148,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kKStages; ++s) {
             tc::mbar_init(KFULL(s), 1);
-            tc::mbar_init(VFULL(s), 1);
             tc::mbar_init(KEMPTY(s), 1);
+        }
+        for (int s = 0; s < kVStages; ++s) {
+            tc::mbar_init(VFULL(s), 1);
             tc::mbar_init(VEMPTY(s), 1);
         }
         for (int w = 0; w < 2; ++w) {
             tc::mbar_init(SFULL(w), 1);
-            tc::mbar_init(SFREE(w), kRows);
-            for (int b = 0; b < 2; ++b) {
-                tc::mbar_init(PFULL(w, b), kRows);
-                tc::mbar_init(PVDONE(w, b), 1);
-            }
+            tc::mbar_init(PFULL(w), kRows);
+            tc::mbar_init(ODONE(w), 1);
+            tc::mbar_init(OFREE(w), kRows);
             tc::mbar_init(ITEMFULL(w), 1);
-            tc::mbar_init(ITEMEMPTY(w), 3 + 2 * kRows);  // two MMA issuers, V producer, 256 softmax rows
+            tc::mbar_init(ITEMEMPTY(w), 2 + 2 * kRows);  // MMA issuer, V producer, 256 softmax rows
         }
         tc::mbar_init(QFULL, 1);
         tc::mbar_init(QEMPTY, 1);
         tc::mbar_init(VZERO, 1);
-        tc::mbar_init(DRAIN(0), 1);
-        tc::mbar_init(DRAIN(1), 1);
+        tc::mbar_init(DRAIN, 1);
         *abort_flag = 0;
         tc::fence_mbar_init();
     }
@@ -182,6 +188,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         return false;
     };
 
+    if (warp >= 8) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsHelper));
     if (warp == 8 || warp == 9) {
         // ---------------------------------- producers (8: scheduler, Q, K; 9: V)
         const bool is_k = warp == 8;
@@ -190,9 +198,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (is_k) tc::prefetch_tmap(&maps.q);
         }
         const int bs = p.block_size;
-        const int per_tile = kKeys / bs;
+        const int per_tile = kKeys / bs;  // blocks per tile (<= 8)
+        const int nst = is_k ? kKStages : kVStages;
         const CUtensorMap *map = is_k ? &maps.k : &maps.v;
-        int g = 0;  // tiles issued so far (stage ring position)
+        int g = 0;  // tiles issued so far (ring position)
         int nfix = 0;
         for (int k = 0;; ++k) {
             const int slot = k & 1;
@@ -232,19 +241,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             int blk_next = (lane < per_tile && b00 + lane < nblk_seq) ? __ldg(bt + b00 + lane) : 0;
             bool ok = true;
             for (int i = 0; i < it.ntiles; ++i, ++g) {
-                const int st = g % kStages;
+                const int st = g % nst;
                 const int blk_cur = blk_next;
                 const int jn = b00 + (i + 1) * per_tile + lane;
                 blk_next = (i + 1 < it.ntiles && lane < per_tile && jn < nblk_seq) ? __ldg(bt + jn) : 0;
-                if (g >= kStages && !wait(is_k ? KEMPTY(st) : VEMPTY(st), ((g / kStages) - 1) & 1)) { ok = false; break; }
+                if (g >= nst && !wait(is_k ? KEMPTY(st) : VEMPTY(st), ((g / nst) - 1) & 1)) { ok = false; break; }
                 int nvalid = nblk_seq - b00 - i * per_tile;
                 nvalid = nvalid < 0 ? 0 : (nvalid > per_tile ? per_tile : nvalid);
                 nvalid = __shfl_sync(0xffffffffu, nvalid, 0);
-                const uint32_t dst = s_base + st * Cfg::kStageBytes + (is_k ? 0 : Cfg::kTileBytes);
+                const uint32_t dst = s_base + (is_k ? 0 : Cfg::kVOff) + st * Cfg::kTileBytes;
                 const uint32_t bar = is_k ? KFULL(st) : VFULL(st);
                 tc::mbar_arrive_expect_tx_warp(bar, static_cast<uint32_t>(nvalid) * bs * D * 2);
-#pragma unroll
-                for (int b = 0; b < 4; ++b) {
+                for (int b = 0; b < per_tile; ++b) {
                     const int blk = __shfl_sync(0xffffffffu, blk_cur, b);
                     if (b < nvalid) {
 #pragma unroll
@@ -254,13 +262,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (!is_k && i == it.ntiles - 1 && it.tail_fix) {
                     // zero V rows of keys >= ctx (stale slots, unloaded blocks)
-                    if (!wait(VFULL(st), (g / kStages) & 1)) { ok = false; break; }
+                    if (!wait(VFULL(st), (g / nst) & 1)) { ok = false; break; }
                     const int r0 = it.ctx - (it.kt0 + i) * kKeys;
                     const int nrows = kKeys - r0;
                     for (int e = lane; e < nrows * 8 * (D / 64); e += 32) {
                         const int h = e / (nrows * 8), rem = e % (nrows * 8);
                         const int row = r0 + rem / 8, ch = rem % 8;
-                        *reinterpret_cast<uint4 *>(smem + st * Cfg::kStageBytes + Cfg::kTileBytes + h * Cfg::kHalf +
+                        *reinterpret_cast<uint4 *>(smem + Cfg::kVOff + st * Cfg::kTileBytes + h * Cfg::kHalf +
                                                    row * 128 + ch * 16) = make_uint4(0u, 0u, 0u, 0u);
                     }
                     tc::fence_proxy_async_smem();
@@ -272,23 +280,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             if (!is_k) tc::mbar_arrive_warp(ITEMEMPTY(slot));
         }
-    } else if (warp == 10 || warp == 11) {
-        // ------------------------------------------------------- MMA issuers
-        // Each warp runs its loop with warp-uniform values (passed through
-        // __shfl_sync so the compiler keeps them in uniform registers); each
-        // tcgen05 instruction is issued by one elected lane. Warp 10 issues the
-        // S products, warp 11 the PV products; tcgen05.commit tracks only the
-        // issuing warp's own MMAs, so each warp commits its own barriers.
-        const bool s_issuer = warp == 10;
+    } else if (warp == 10) {
+        // -------------------------------------------------------- MMA issuer
+        // The loop runs with warp-uniform values (passed through __shfl_sync
+        // so the compiler keeps them in uniform registers); each tcgen05
+        // instruction is issued by one elected lane.
         constexpr uint32_t idS = tc::idesc_bf16(kRows, kKeys, false);
         constexpr uint32_t idO = tc::idesc_bf16(kRows, D, true);
         const uint32_t utmem = __shfl_sync(0xffffffffu, tmem, 0);
         const uint32_t us_base = __shfl_sync(0xffffffffu, s_base, 0);
-        int g = 0, t = 0, nfix = 0;
+        int gk = 0, gv = 0, t = 0, nfix = 0;
         bool ok = true, issued = false;
         auto issue_s = [&](int w, int st_in) {
             const int st = __shfl_sync(0xffffffffu, st_in, 0);
-            const uint64_t kd = tc::sdesc_sw128(us_base + st * Cfg::kStageBytes, 16, 1024);
+            const uint64_t kd = tc::sdesc_sw128(us_base + st * Cfg::kTileBytes, 16, 1024);
             const uint64_t qd = tc::sdesc_sw128(us_base + Cfg::kQOff + w * Cfg::kQBytes, 16, 1024);
             const uint32_t dS = utmem + col_s(w);
 #pragma unroll
@@ -296,17 +301,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::mma_ss_warp(dS, qd + ((kk / 4) * Cfg::kQHalf + (kk % 4) * 32) / 16,
                                 kd + ((kk / 4) * Cfg::kHalf + (kk % 4) * 32) / 16, idS, kk > 0);
             tc::commit_warp(SFULL(w));
+            issued = true;
         };
-        auto issue_pv = [&](int w, int st_in, int b_in, uint32_t acc_in) {
+        auto issue_pv = [&](int w, int st_in, uint32_t acc_in) {
             const int st = __shfl_sync(0xffffffffu, st_in, 0);
-            const int b = __shfl_sync(0xffffffffu, b_in, 0);
             const uint32_t acc = __shfl_sync(0xffffffffu, acc_in, 0);
-            const uint64_t vd = tc::sdesc_sw128(us_base + st * Cfg::kStageBytes + Cfg::kTileBytes, Cfg::kHalf, 1024);
-            const uint32_t dO = utmem + col_o(w), aP = utmem + col_p(w, 0) + 32u * b;
+            const uint64_t vd =
+                tc::sdesc_sw128(us_base + Cfg::kVOff + st * Cfg::kTileBytes, Cfg::kHalf, 1024);
+            const uint32_t dO = utmem + col_o(w), aP = utmem + col_s(w);
             tc::mma_ts_warp(dO, aP, vd, idO, acc);
 #pragma unroll
             for (int kk = 1; kk < kKeys / 16; ++kk) tc::mma_ts_warp(dO, aP + kk * 8, vd + (kk * 2048) / 16, idO, 1u);
-            tc::commit_warp(PVDONE(w, b));
+            issued = true;
         };
         for (int k = 0; ok; ++k) {
             const int slot = k & 1;
@@ -316,52 +322,62 @@ __global__ void __launch_bounds__(kThreads, 1)
             const ItemGeom it = item_geom(p, idx);
             const int n = __shfl_sync(0xffffffffu, it.ntiles, 0);
             const bool tail = __shfl_sync(0xffffffffu, it.tail_fix ? 1 : 0, 0) != 0;
-            if (s_issuer) {
-                if (!wait(QFULL, k & 1)) { ok = false; break; }
-                for (int j = 0; j < n; ++j) {
-                    const int T = t + j, gj = g + j, st = gj % kStages;
-                    if (!wait(KFULL(st), (gj / kStages) & 1)) { ok = false; break; }
-                    // S_w(T) overwrites S_w(T - 1), which warpgroup w has copied out
-                    if (T >= 1 && !wait(SFREE(0), (T - 1) & 1)) { ok = false; break; }
-                    tc::fence_after_sync();
-                    issue_s(0, st);
-                    issued = true;
-                    if (T >= 1 && !wait(SFREE(1), (T - 1) & 1)) { ok = false; break; }
-                    tc::fence_after_sync();
-                    issue_s(1, st);
-                    tc::commit_warp(KEMPTY(st));
-                    if (j == n - 1) tc::commit_warp(QEMPTY);  // last S of this item
+            // S_0(0), S_1(0)
+            if (!wait(QFULL, k & 1)) { ok = false; break; }
+            if (!wait(KFULL(gk % kKStages), (gk / kKStages) & 1)) { ok = false; break; }
+            tc::fence_after_sync();
+            issue_s(0, gk % kKStages);
+            issue_s(1, gk % kKStages);
+            tc::commit_warp(KEMPTY(gk % kKStages));
+            ++gk;
+            if (n == 1) tc::commit_warp(QEMPTY);
+            for (int j = 0; j < n; ++j) {
+                const int T = t + j, vst = gv % kVStages;
+                if (j == n - 1 && tail) {
+                    if (!wait(VZERO, nfix & 1)) { ok = false; break; }
+                } else if (!wait(VFULL(vst), (gv / kVStages) & 1)) {
+                    ok = false;
+                    break;
                 }
-            } else {
-                for (int j = 0; j < n; ++j) {
-                    const int T = t + j, gj = g + j, st = gj % kStages;
-                    if (j == n - 1 && tail) {
-                        if (!wait(VZERO, nfix & 1)) { ok = false; break; }
-                    } else if (!wait(VFULL(st), (gj / kStages) & 1)) {
-                        ok = false;
-                        break;
-                    }
-                    if (!wait(PFULL(0, T & 1), (T >> 1) & 1)) { ok = false; break; }
+                // O_0 += P_0(j) V(j), then S_0(j + 1)
+                if (!wait(PFULL(0), T & 1)) { ok = false; break; }
+                if (j == 0 && k >= 1 && !wait(OFREE(0), (k - 1) & 1)) { ok = false; break; }
+                tc::fence_after_sync();
+                issue_pv(0, vst, j > 0 ? 1u : 0u);
+                if (j == n - 1) tc::commit_warp(ODONE(0));
+                const bool more = j + 1 < n;
+                if (more) {
+                    if (!wait(KFULL(gk % kKStages), (gk / kKStages) & 1)) { ok = false; break; }
                     tc::fence_after_sync();
-                    issue_pv(0, st, T & 1, j > 0 ? 1u : 0u);
-                    issued = true;
-                    if (!wait(PFULL(1, T & 1), (T >> 1) & 1)) { ok = false; break; }
-                    tc::fence_after_sync();
-                    issue_pv(1, st, T & 1, j > 0 ? 1u : 0u);
-                    tc::commit_warp(VEMPTY(st));
+                    issue_s(0, gk % kKStages);
+                }
+                // O_1 += P_1(j) V(j), then S_1(j + 1)
+                if (!wait(PFULL(1), T & 1)) { ok = false; break; }
+                if (j == 0 && k >= 1 && !wait(OFREE(1), (k - 1) & 1)) { ok = false; break; }
+                tc::fence_after_sync();
+                issue_pv(1, vst, j > 0 ? 1u : 0u);
+                tc::commit_warp(VEMPTY(vst));
+                ++gv;
+                if (j == n - 1) tc::commit_warp(ODONE(1));
+                if (more) {
+                    issue_s(1, gk % kKStages);
+                    tc::commit_warp(KEMPTY(gk % kKStages));
+                    ++gk;
+                    if (j + 1 == n - 1) tc::commit_warp(QEMPTY);  // last S of this item
                 }
             }
             if (!ok) break;
-            g += n;
             t += n;
             if (tail) ++nfix;
             tc::mbar_arrive_warp(ITEMEMPTY(slot));
         }
-        if (!ok && issued) {  // drain whatever this warp still has in flight
-            tc::commit_warp(DRAIN(s_issuer ? 0 : 1));
-            tc::mbar_wait(DRAIN(s_issuer ? 0 : 1), 0, 200000000ull);
+        if (!ok && issued) {  // drain whatever is still in flight
+            tc::commit_warp(DRAIN);
+            tc::mbar_wait(DRAIN, 0, 200000000ull);
         }
+    }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsSoftmax));
         // ------------------------------------------- softmax / epilogue rows
         const int w = warp >> 2;                 // warpgroup = Q tile
         const int r = tid & 127;                 // MMA row = TMEM lane
@@ -388,39 +404,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             float l = 0.f;
             bool ok = true;
             for (int i = 0; i < it.ntiles; ++i) {
-                const int T = t + i, b = T & 1;
+                const int T = t + i;
                 if (!wait(SFULL(w), T & 1)) { ok = false; break; }
                 tc::fence_after_sync();
-                uint32_t s[64];
-                tc::tmem_ld32(lane_addr + col_s(w), *reinterpret_cast<uint32_t(*)[32]>(&s[0]));
-                tc::tmem_ld32(lane_addr + col_s(w) + 32, *reinterpret_cast<uint32_t(*)[32]>(&s[32]));
+                uint32_t s[kKeys];
+#pragma unroll
+                for (int c = 0; c < kKeys / 32; ++c)
+                    tc::tmem_ld32(lane_addr + col_s(w) + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&s[32 * c]));
                 tc::tmem_wait_ld();
-                tc::fence_before_sync();
-                tc::mbar_arrive(SFREE(w));  // the S buffer may be overwritten now
                 // tiles that reach past the first row's position need the causal
                 // mask; all others are fully visible to every row of the tile
                 const int k0 = (it.kt0 + i) * kKeys;
                 const bool masked_tile = k0 + kKeys - 1 > min_pos;
-                float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
                 if (masked_tile) {
 #pragma unroll
-                    for (int j = 0; j < kKeys; j += 4) {
-                        float v0 = __uint_as_float(s[j]), v1 = __uint_as_float(s[j + 1]);
-                        float v2 = __uint_as_float(s[j + 2]), v3 = __uint_as_float(s[j + 3]);
-                        v0 = (k0 + j <= pos) ? v0 : -INFINITY;
-                        v1 = (k0 + j + 1 <= pos) ? v1 : -INFINITY;
-                        v2 = (k0 + j + 2 <= pos) ? v2 : -INFINITY;
-                        v3 = (k0 + j + 3 <= pos) ? v3 : -INFINITY;
-                        s[j] = __float_as_uint(v0); s[j + 1] = __float_as_uint(v1);
-                        s[j + 2] = __float_as_uint(v2); s[j + 3] = __float_as_uint(v3);
-                        mx0 = fmaxf(mx0, v0); mx1 = fmaxf(mx1, v1); mx2 = fmaxf(mx2, v2); mx3 = fmaxf(mx3, v3);
-                    }
-                } else {
+                    for (int j = 0; j < kKeys; ++j)
+                        if (k0 + j > pos) s[j] = __float_as_uint(-INFINITY);
+                }
+                float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
 #pragma unroll
-                    for (int j = 0; j < kKeys; j += 4) {
-                        mx0 = fmaxf(mx0, __uint_as_float(s[j])); mx1 = fmaxf(mx1, __uint_as_float(s[j + 1]));
-                        mx2 = fmaxf(mx2, __uint_as_float(s[j + 2])); mx3 = fmaxf(mx3, __uint_as_float(s[j + 3]));
-                    }
+                for (int j = 0; j < kKeys; j += 8) {
+                    mx0 = fmax3(mx0, __uint_as_float(s[j]), __uint_as_float(s[j + 1]));
+                    mx1 = fmax3(mx1, __uint_as_float(s[j + 2]), __uint_as_float(s[j + 3]));
+                    mx2 = fmax3(mx2, __uint_as_float(s[j + 4]), __uint_as_float(s[j + 5]));
+                    mx3 = fmax3(mx3, __uint_as_float(s[j + 6]), __uint_as_float(s[j + 7]));
                 }
                 // the scale is positive, so the max of scaled scores is the scaled max
                 const float tmax = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sc;
@@ -428,9 +435,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (__any_sync(0xffffffffu, need)) {
                     const float m_new = need ? fmaxf(m_run, tmax) : m_run;
                     const float alpha = (need && m_run != -INFINITY) ? fast_exp2(m_run - m_new) : 1.f;
-                    if (i > 0) {  // rescale O_w once PV_w of the previous tile has landed
-                        if (!wait(PVDONE(w, (T - 1) & 1), ((T - 1) >> 1) & 1)) { ok = false; break; }
-                        tc::fence_after_sync();
+                    if (i > 0) {
+                        // PV_w(i - 1) is complete: S_w(i) was issued after it
 #pragma unroll
                         for (int c = 0; c < D / 32; ++c) {
                             uint32_t o[32];
@@ -445,29 +451,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                     m_run = m_new;
                 }
                 const float nbase = (m_run == -INFINITY) ? 0.f : -m_run;
-                // P buffer b last held P(T - 2): wait until PV(T - 2) has read it
-                if (T >= 2 && !wait(PVDONE(w, b), ((T - 2) >> 1) & 1)) { ok = false; break; }
-                float l0 = 0.f, l1 = 0.f;
+                // x = s * scale - m and the row sum on paired fp32 lanes
+                const uint64_t sc2 = f2_pack(sc, sc), nb2 = f2_pack(nbase, nbase);
+                uint64_t lacc0 = f2_pack(0.f, 0.f), lacc1 = lacc0;
 #pragma unroll
-                for (int hlf = 0; hlf < 2; ++hlf) {
+                for (int q4 = 0; q4 < kKeys / 32; ++q4) {
                     uint32_t pk[16];
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        const float p0 = fast_exp2(fmaf(__uint_as_float(s[32 * hlf + 2 * j]), sc, nbase));
-                        const float p1 = fast_exp2(fmaf(__uint_as_float(s[32 * hlf + 2 * j + 1]), sc, nbase));
-                        if (j & 1) l1 += p0 + p1; else l0 += p0 + p1;
+                        const uint64_t x2 = f2_fma(f2_pack(__uint_as_float(s[32 * q4 + 2 * j]),
+                                                           __uint_as_float(s[32 * q4 + 2 * j + 1])), sc2, nb2);
+                        float x0, x1;
+                        f2_unpack(x2, x0, x1);
+                        const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+                        if (j & 1) lacc1 = f2_add(lacc1, f2_pack(p0, p1));
+                        else lacc0 = f2_add(lacc0, f2_pack(p0, p1));
                         pk[j] = pack_bf16x2(p0, p1);
                     }
-                    tc::tmem_st16(lane_addr + col_p(w, b) + 16 * hlf, pk);
+                    tc::tmem_st16(lane_addr + col_s(w) + 16 * q4, pk);
                 }
-                l += l0 + l1;
+                {
+                    float a0, a1;
+                    f2_unpack(f2_add(lacc0, lacc1), a0, a1);
+                    l += a0 + a1;
+                }
                 tc::tmem_wait_st();
                 tc::fence_before_sync();
-                tc::mbar_arrive(PFULL(w, b));
+                tc::mbar_arrive(PFULL(w));
             }
             if (!ok) break;
-            const int Tl = t + it.ntiles - 1;
-            if (!wait(PVDONE(w, Tl & 1), (Tl >> 1) & 1)) break;
+            if (!wait(ODONE(w), k & 1)) break;
             tc::fence_after_sync();
             const float inv = 1.f / l;
             uint4 *orow = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
@@ -576,6 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             t += it.ntiles;
             tc::fence_before_sync();
+            tc::mbar_arrive(OFREE(w));  // O_w may be overwritten by the next item
             tc::mbar_arrive(ITEMEMPTY(slot));
         }
     }
@@ -672,6 +686,9 @@ bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group) {
 
 // positions per work item: two Q tiles of floor(128 / G) positions each
 int prefill_tc_rows_per_item(int group) { return 2 * (kRows / group); }
+
+// keys per K/V tile (the unit of the planner's key splits)
+int prefill_tc_keys_per_tile() { return kKeys; }
 
 int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas) {
     if (p.num_pitems == 0) return FNPU_OK;
