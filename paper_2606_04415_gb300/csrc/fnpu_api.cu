@@ -81,26 +81,33 @@ void destroy_sync_objects(fnpu_plan *pl) {
     pl->e_fork = pl->e_pre = pl->e_dec = nullptr;
 }
 
-// Modelled rates of the two phases: a prefill CTA finishes one 128-key tile
-// of both Q tiles (d = 128) in about 1.6 us; a decode SM streams about 60 GB/s
-// of KV cache and the whole device about 4 TB/s.
-constexpr double kTileSec = 1.6e-6;
-constexpr double kDecodeSmBps = 60e9;
+// Modelled rates of the two phases (measured on the co-located Qwen2.5-7B
+// step): a prefill CTA finishes one 128-key tile of both Q tiles (d = 128)
+// in about 1.5 us; a decode SM streams about 69 GB/s of KV cache and the
+// whole device about 4 TB/s.
+constexpr double kTileSec = 1.5e-6;
+constexpr double kDecodeSmBps = 69e9;
 constexpr double kDecodeAllBps = 4.0e12;
 
-// SMs that start on decode while the others run prefill: prefill on sms - k
-// SMs lasts Tp; decode streams at min(all, k * per SM) meanwhile, and what is
+int64_t lpt_makespan(const std::vector<int64_t> &costs, int32_t m);
+
+// SMs that start on decode while the others run prefill: the prefill CTAs on
+// sms - k SMs take the items longest first, so they last about the LPT
+// makespan Tp of the item costs on sms - k workers (a step function of k:
+// whole items); decode streams at min(all, k * per SM) meanwhile, and what is
 // left runs on every SM once the prefill CTAs have finished. The k with the
-// shortest modelled step wins.
-int32_t choose_decode_sms(int64_t pre_tiles, int64_t dec_bytes, int32_t sms) {
+// shortest modelled step wins, the largest such k on ties (more decode done
+// while the prefill lasts).
+int32_t choose_decode_sms(const std::vector<int64_t> &item_tiles, double tile_scale, int64_t dec_bytes,
+                          int32_t sms) {
     int32_t best_k = 1;
     double best_t = -1.0;
     for (int32_t k = 1; k <= sms / 2; ++k) {
-        const double tp = static_cast<double>(pre_tiles) * kTileSec / (sms - k);
+        const double tp = static_cast<double>(lpt_makespan(item_tiles, sms - k)) * tile_scale * kTileSec;
         const double rate = std::min(kDecodeAllBps, k * kDecodeSmBps);
         const double left = std::max(0.0, static_cast<double>(dec_bytes) - tp * rate);
         const double t = tp + left / kDecodeAllBps;
-        if (best_t < 0 || t < best_t) {
+        if (best_t < 0 || t <= best_t) {
             best_t = t;
             best_k = k;
         }
@@ -390,8 +397,11 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 }
             }
         } else if (phase[s] == 1 && pl->use_dt) {
-            // items over all kv heads; one merge counter per (sequence, kv head)
-            const int32_t sk = std::max(split, (c + 255 * 64) / (256 * 64) * 64);
+            // items over all kv heads; one merge counter per (sequence, kv head).
+            // At most 16 splits per sequence: the last split merges them, with
+            // one memory round trip per two splits, and a long sequence's merge
+            // would otherwise end the step late
+            const int32_t sk = std::max(split, (c + 16 * 64 - 1) / (16 * 64) * 64);
             const int32_t ns = (c + sk - 1) / sk;
             const int32_t grp = groups;
             groups += desc->num_kv_heads;
@@ -446,12 +456,13 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         for (const DecodeItem &it : ditems)
             dec_bytes += static_cast<int64_t>(it.key_end - it.key_begin) * desc->num_kv_heads *
                          (desc->head_dim_qk + desc->head_dim_v) * 2;
-        int64_t pre_tiles = 0;
-        for (const TcUnit &u : tc_units) pre_tiles += u.ntiles + kTcItemCost;
-        pre_tiles = pre_tiles * (desc->head_dim_qk + desc->head_dim_v) / 256;  // in d = 128 tiles
+        std::vector<int64_t> item_tiles;
+        for (const TcUnit &u : tc_units) item_tiles.push_back(u.ntiles + kTcItemCost);
+        std::sort(item_tiles.begin(), item_tiles.end(), [](int64_t a, int64_t b) { return a > b; });
+        const double tile_scale = (desc->head_dim_qk + desc->head_dim_v) / 256.0;  // relative to d = 128
         const int32_t k = o.decode_share_pct > 0
                               ? std::min(sms - 1, std::max(1, (sms * o.decode_share_pct + 50) / 100))
-                              : choose_decode_sms(pre_tiles, dec_bytes, sms);
+                              : choose_decode_sms(item_tiles, tile_scale, dec_bytes, sms);
         pl->pre_ctas = sms - k;
     }
     int32_t pparts = 0, pgroups = 0;
