@@ -51,8 +51,10 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    // one pass over all chunks when it fits 32 blocks per SM: the copy is
+    // latency-bound at step sizes, so every chunk should be in flight at once
     const int64_t want = (total + 255) / 256;
-    const int grid = static_cast<int>(want < 8LL * sms ? want : 8LL * sms);
+    const int grid = static_cast<int>(want < 32LL * sms ? want : 32LL * sms);
     kv_append_kernel<<<grid, 256, 0, static_cast<cudaStream_t>(stream)>>>(
         static_cast<const uint4 *>(k_new), static_cast<const uint4 *>(v_new), slots, num_tokens,
         kc, vc, static_cast<uint4 *>(k_cache), static_cast<uint4 *>(v_cache),
