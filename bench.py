@@ -86,6 +86,24 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(value, ws, device):
+    """The largest of each rank's value: a job's step time is its slowest
+    replica's. Every rank gets the same result."""
+    if ws <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(ws, tokens_per_rank, ms):
+    """Whole-job query tokens/s: every replica processes its own batch of
+    tokens_per_rank tokens in the job's step time (weak scaling)."""
+    return ws * tokens_per_rank / (ms * 1e-3)
+
+
 class ClockSampler:
     """nvidia-smi clocks/throttle reasons sampled every 200 ms while active."""
 
@@ -266,12 +284,8 @@ def run_fnpu(args):
     clk = clocks.summary()
     t_append = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
     t_attn = [ev[i][1].elapsed_time(ev[i][2]) for i in range(K)]
-    step_ms = sum(a + b for a, b in zip(t_append, t_attn)) / K
+    step_ms = max_over_ranks(sum(a + b for a, b in zip(t_append, t_attn)) / K, ws, dev)
     attn_ms = sum(t_attn) / K
-    if ws > 1:
-        t = torch.tensor([step_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        step_ms = float(t.item())
 
     # end to end through host buffers: H2D of the step's inputs, append + attention,
     # D2H of the outputs, all inside the timed region
@@ -302,11 +316,7 @@ def run_fnpu(args):
         b.synchronize()
         if i >= args.warmup:
             e2e_ms.append(a.elapsed_time(b))
-    e2e = sum(e2e_ms) / len(e2e_ms)
-    if ws > 1:
-        t = torch.tensor([e2e], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e = float(t.item())
+    e2e = max_over_ranks(sum(e2e_ms) / len(e2e_ms), ws, dev)
 
     # roofline of the dominant kernel work (the attention launch): algorithmic
     # FLOPs and bytes per run / measured duration
@@ -328,7 +338,7 @@ def run_fnpu(args):
 
     T = batch.num_tokens
     line = {
-        "metric": METRIC, "value": ws * T / (step_ms * 1e-3), "unit": UNIT, "n_gpus": ws,
+        "metric": METRIC, "value": job_throughput(ws, T, step_ms), "unit": UNIT, "n_gpus": ws,
         "steps": K, "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T,
@@ -340,7 +350,7 @@ def run_fnpu(args):
                                "sustained": step_roof_sus / (step_ms * 1e-3),
                                "denominator": "max(F/bf16 peak, B/HBM peak) of measured"},
         "kernel_ms": {"append": sum(t_append) / K, "attention": attn_ms},
-        "e2e": {"value": ws * T / (e2e * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
         "gpu_launches": K * (1 + info["launches_per_run"]),
         "clocks": clk,
