@@ -102,6 +102,46 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     return r;
 }
 
+// Programmatic dependent launch: the trigger lets a kernel launched after this
+// one on the same stream (with programmatic serialization) start once every CTA
+// of this grid has issued it; the wait blocks until the grids this one depends
+// on have completed and their writes are visible (a no-op without a dependency).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+
+// Kernel launch with the two ordering options the step uses: `after_prev`
+// lets the kernel start before the previous kernel on the stream has ended
+// (programmatic dependent launch: it is released once every CTA of that grid
+// has triggered or ended, and a pdl_wait() in it waits for that grid's
+// writes); `started`, if not null, is recorded once every CTA of this grid
+// has begun (a launch completion event; the runtime treats it as best
+// effort, and at worst it fires when the grid ends).
+template <typename... Args>
+cudaError_t launch_ex(void (*kernel)(Args...), int grid, int threads, size_t smem, cudaStream_t st, bool after_prev,
+                      cudaEvent_t started, const Args &...args) {
+    cudaLaunchAttribute attr[2];
+    int n = 0;
+    if (after_prev) {
+        attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (started) {
+        attr[n].id = cudaLaunchAttributeLaunchCompletionEvent;
+        attr[n].val.launchCompletionEvent.event = started;
+        attr[n].val.launchCompletionEvent.flags = 0;
+        ++n;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = n;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 

@@ -3,16 +3,19 @@
 // size a multiple of 16).
 //
 // Decode is bound by KV-cache reads (Sec. 1, Sec. 3.3, Fig. 2). The kernel is
-// kept small -- four warps, at most 128 registers a thread, 64 KB of shared
-// memory for d = 128 -- so that up to three CTAs share an SM and a few SMs
-// alone can stream decode work while the others run prefill (Sec. 3.4).
+// kept small -- five warps, at most 128 registers a thread, 64 KB of shared
+// memory for d = 128 -- so that three CTAs share an SM and a few SMs alone
+// can stream decode work while the others run prefill (Sec. 3.4).
 //   * Persistent CTAs take items -- a sequence's key range, longest first --
-//     from an atomic queue two items ahead of use (the last CTA out resets it);
+//     from an atomic queue one item ahead of use (the last CTA out resets it);
 //     the next item's descriptor, block ids and query are loaded during the
-//     current item, so an item boundary costs no memory round trip.
-//   * A 2-stage ring of 16-key stages holds K and V of all four kv heads. Warp
-//     0 issues the TMA copies of the stage after the one it is about to read:
-//     four boxes of 16 slots x 4 heads x 64 columns for d = 128. The tensor map
+//     current item, so an item boundary costs no memory round trip. (Taking
+//     two items ahead left CTAs idle when items were few: the first CTAs
+//     reserved them all.)
+//   * A 2-stage ring of 16-key stages holds K and V of all four kv heads. A
+//     producer warp issues the TMA copies (four boxes of 16 slots x 4 heads x
+//     64 columns for d = 128) as soon as a stage is free; issuing them from a
+//     compute warp cost that warp about as much as its arithmetic. The tensor map
 //     lists the slot dimension before the kv-head dimension, so a box lands
 //     head-major (16 consecutive slots of one head form 16 rows) and the
 //     128-byte swizzle is keyed by the slot: ldmatrix over eight consecutive
@@ -23,10 +26,11 @@
 //   * V rows past the item's keys are zeroed by their warp before the PV
 //     product, so stale slots never reach it.
 //   * A split writes its partial result (Eq. 1 restricted to its keys, with
-//     its log-sum-exp); the last split of a (sequence, kv head) to finish
-//     merges all of them. The release fence and the counter update of an item
-//     are deferred to the second stage of the next item, when the partial
-//     stores have long completed, and a merge they trigger to the end of it.
+//     its log-sum-exp); a second small kernel merges the splits of every
+//     sequence, one warp per (token, query head), all in parallel. Merging in
+//     the last split instead took one dependent round trip per two splits and
+//     capped the splits per sequence, and with few splits the items were too
+//     coarse to share the bandwidth evenly among the CTAs.
 // Every mbarrier wait is bounded and raises the plan's error flag on timeout.
 #include <math.h>
 
@@ -41,8 +45,8 @@ namespace {
 constexpr int kHkv = 4;
 constexpr int kKeys = 16;        // keys per stage
 constexpr int kStages = 2;
-constexpr int kWarps = 4;        // one per kv head
-constexpr int kThreads = 32 * kWarps;
+constexpr int kWarps = 4;        // compute warps, one per kv head
+constexpr int kThreads = 32 * (kWarps + 1);  // + the TMA producer warp
 constexpr int kHalfBytes = kHkv * kKeys * 128;  // all heads, one 64-column half
 
 template <int D>
@@ -50,8 +54,8 @@ struct DtCfg {
     static constexpr int kTileBytes = (D / 64) * kHalfBytes;  // K or V of one stage
     static constexpr int kStageBytes = 2 * kTileBytes;
     static constexpr int kBarOff = kStages * kStageBytes;
-    // full[S] empty[S] itemdone[2]
-    static constexpr int kNumBars = 2 * kStages + 2;
+    // full[S] empty[S]
+    static constexpr int kNumBars = 2 * kStages;
     // + item ring [4] and the abort flag
     static constexpr int kSmemBytes = kBarOff + 8 * kNumBars + 32;
 };
@@ -98,7 +102,7 @@ __device__ __forceinline__ int load_blk_lane(const AttnParams &p, const DtGeo &g
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 4)
+__global__ void __launch_bounds__(kThreads, 3)
     decode_tma_kernel(const AttnParams p, const __grid_constant__ DtMaps maps) {
     using Cfg = DtCfg<D>;
     extern __shared__ __align__(1024) uint8_t smem[];
@@ -106,13 +110,13 @@ __global__ void __launch_bounds__(kThreads, 4)
     const uint32_t s_bars = s_base + Cfg::kBarOff;
     auto FULL = [&](int s) { return s_bars + 8 * s; };
     auto EMPTY = [&](int s) { return s_bars + 8 * (kStages + s); };
-    auto ITEMDONE = [&](int b) { return s_bars + 8 * (2 * kStages + b); };
     int *ring = reinterpret_cast<int *>(smem + Cfg::kBarOff + 8 * Cfg::kNumBars);  // [4]
     volatile int *abort_flag = ring + 4;
     int *sched = p.sched + 2;  // this kernel's work queue: next item, finished CTAs
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n_items = p.num_ditems;
+    pdl_trigger();  // the merge grid may be placed once these CTAs are; it waits for them to finish
     if ((s_base & 1023u) != 0) {  // the swizzled tiles need 1024-byte alignment
         if (tid == 0) atomicOr(p.err, 2);
         return;
@@ -122,14 +126,11 @@ __global__ void __launch_bounds__(kThreads, 4)
             tc::mbar_init(FULL(s), 1);
             tc::mbar_init(EMPTY(s), kWarps);
         }
-        tc::mbar_init(ITEMDONE(0), kWarps);
-        tc::mbar_init(ITEMDONE(1), kWarps);
         ring[0] = atomicAdd(sched, 1);
-        ring[1] = atomicAdd(sched, 1);
         *abort_flag = 0;
         tc::fence_mbar_init();
     }
-    if (warp == 0 && lane == 0) {
+    if (warp == kWarps && lane == 0) {
         tc::prefetch_tmap(&maps.k);
         tc::prefetch_tmap(&maps.v);
     }
@@ -164,7 +165,7 @@ __global__ void __launch_bounds__(kThreads, 4)
     const int bs = p.block_size;
     __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
 
-    // issue stage `j` of item `g` into ring position `gs` (warp 0, whole warp)
+    // issue stage `j` of item `g` into ring position `gs` (producer warp, whole warp)
     auto issue = [&](const DtGeo &g, int j, int blk_lane, int gs) -> bool {
         const int st = gs % kStages;
         if (gs >= kStages && !wait(EMPTY(st), ((gs / kStages) - 1) & 1)) return false;
@@ -182,92 +183,58 @@ __global__ void __launch_bounds__(kThreads, 4)
         return true;
     };
 
-    // merge of the splits of (sequence of token t, this kv head), by the last split
-    auto merge = [&](int t, int ns, int base) {
-        float M[8], L[8];
-#pragma unroll
-        for (int h = 0; h < 8; ++h) { M[h] = -INFINITY; L[h] = 0.f; }
-        for (int sp = lane; sp < ns; sp += 32) {
-            const float *pl = p.part_lse + static_cast<int64_t>(base + sp) * Hq + head * G;
-#pragma unroll
-            for (int h = 0; h < 8; ++h)
-                if (h < G) M[h] = fmaxf(M[h], __ldcg(pl + h));
+    if (warp == kWarps) {
+        // ---------------------------------------------------- TMA producer
+        // Runs up to kStages stages ahead of the compute warps. It takes the
+        // next item from the queue at the start of the current one (one item
+        // ahead, so that the queue still balances the CTAs), publishes its
+        // index in the item ring before it issues stage 2 of the current item
+        // (the compute warps read it after that stage has landed), and loads
+        // the next item's descriptor, sequence row and block ids one stage
+        // apart, so that no dependent memory round trip sits between stages.
+        int gs = 0;
+        bool ok = true;
+        int idx = ring[0];
+        DecodeItem it{};
+        SeqInfo si{};
+        if (idx < n_items) {
+            it = p.ditems[idx];
+            si = p.seqs[it.seq];
         }
-#pragma unroll
-        for (int h = 0; h < 8; ++h)
-#pragma unroll
-            for (int o2 = 16; o2 > 0; o2 >>= 1) M[h] = fmaxf(M[h], __shfl_xor_sync(0xffffffffu, M[h], o2));
-        for (int sp = lane; sp < ns; sp += 32) {
-            const float *pl = p.part_lse + static_cast<int64_t>(base + sp) * Hq + head * G;
-#pragma unroll
-            for (int h = 0; h < 8; ++h)
-                if (h < G) L[h] += fast_exp2(__ldcg(pl + h) - M[h]);
-        }
-#pragma unroll
-        for (int h = 0; h < 8; ++h)
-#pragma unroll
-            for (int o2 = 16; o2 > 0; o2 >>= 1) L[h] += __shfl_xor_sync(0xffffffffu, L[h], o2);
-        if (lane < D / 4) {
-            float4 acc[8];
-#pragma unroll
-            for (int h = 0; h < 8; ++h) acc[h] = make_float4(0.f, 0.f, 0.f, 0.f);
-            const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
-#pragma unroll 2
-            for (int sp = 0; sp < ns; ++sp) {
-                const int64_t row = static_cast<int64_t>(base + sp) * Hq + head * G;
-#pragma unroll
-                for (int h = 0; h < 8; ++h) {
-                    if (h < G) {
-                        const float w = fast_exp2(__ldcg(p.part_lse + row + h) - M[h]);
-                        const float4 v = __ldcg(po + (row + h) * (D / 4) + lane);
-                        acc[h].x += w * v.x; acc[h].y += w * v.y; acc[h].z += w * v.z; acc[h].w += w * v.w;
-                    }
+        DtGeo cur = geo_of(it, si);
+        int blk_lane = idx < n_items ? load_blk_lane(p, cur, lane) : 0;
+        for (int k = 0; ok && idx < n_items; ++k) {
+            int a = 0;
+            if (lane == 0) a = atomicAdd(sched, 1);  // the next item
+            const int ntiles = (cur.ke - cur.kb + kKeys - 1) / kKeys;
+            const int spub = ntiles > 2 ? 2 : ntiles - 1;
+            const int s1 = spub + 1 < ntiles ? spub + 1 : spub, s2 = spub + 2 < ntiles ? spub + 2 : s1;
+            int idx_n = n_items;
+            DecodeItem nit{};
+            SeqInfo nsi{};
+            DtGeo nxt{};
+            int blk_lane_n = 0;
+            for (int i = 0; i < ntiles; ++i, ++gs) {
+                if (i == spub) {
+                    idx_n = __shfl_sync(0xffffffffu, a, 0);
+                    if (lane == 0) *reinterpret_cast<volatile int *>(ring + ((k + 1) & 3)) = idx_n;
+                    __syncwarp();  // before the arrival of this stage, which releases it
+                    if (idx_n < n_items) nit = p.ditems[idx_n];
+                }
+                if (!issue(cur, i, blk_lane, gs)) { ok = false; break; }
+                if (idx_n < n_items && i == s1) nsi = p.seqs[nit.seq];
+                if (idx_n < n_items && i == s2) {
+                    nxt = geo_of(nit, nsi);
+                    blk_lane_n = load_blk_lane(p, nxt, lane);
                 }
             }
-#pragma unroll
-            for (int h = 0; h < 8; ++h) {
-                if (h < G) {
-                    const float il = 1.f / L[h];
-                    uint2 pk;
-                    pk.x = pack_bf16x2(acc[h].x * il, acc[h].y * il);
-                    pk.y = pack_bf16x2(acc[h].z * il, acc[h].w * il);
-                    *reinterpret_cast<uint2 *>(out + (static_cast<int64_t>(t) * Hq + head * G + h) * D + lane * 4) = pk;
-                }
-            }
+            if (!ok) break;
+            idx = idx_n;
+            cur = nxt;
+            blk_lane = blk_lane_n;
         }
-        if (lane < G) {
-            float Ml = M[0], Ll = L[0];
-#pragma unroll
-            for (int h = 1; h < 8; ++h)
-                if (lane == h) { Ml = M[h]; Ll = L[h]; }
-            p.lse[static_cast<int64_t>(t) * Hq + head * G + lane] = (Ml + log2f(Ll)) * kLn2;
-        }
-    };
-
-    // A finished split's counter update waits until its partial stores have
-    // completed (a stage into the next item); a merge it triggers runs at the
-    // end of that next item, when the accumulators are free.
-    bool pend = false, mrg = false;
-    int pend_t = 0, pend_ns = 0, pend_base = 0, pend_group = 0;
-    auto settle = [&]() {
-        if (!pend) return;
-        pend = false;
-        __threadfence();  // this warp's partial stores before the counter update
-        __syncwarp();
-        int last = 0;
-        if (lane == 0) last = atomicAdd(p.counters + pend_group * kHkv + head, 1) == pend_ns - 1;
-        mrg = __shfl_sync(0xffffffffu, last, 0) != 0;
-    };
-    auto merge_if_last = [&]() {
-        if (!mrg) return;
-        mrg = false;
-        __threadfence();
-        merge(pend_t, pend_ns, pend_base);
-        if (lane == 0) p.counters[pend_group * kHkv + head] = 0;  // ready for the next run
-    };
-
-    int idx = ring[0];
-    if (idx < n_items) {
+    } else if (ring[0] < n_items) {
+        int idx = ring[0];
         DtGeo cur;
         {
             const DecodeItem it = p.ditems[idx];
@@ -275,47 +242,32 @@ __global__ void __launch_bounds__(kThreads, 4)
         }
         uint32_t qb[D / 16][2];
         load_q<D>(p, cur.t, head, g8, c, qb);
-        int blk_lane = warp == 0 ? load_blk_lane(p, cur, lane) : 0;
         bool ok = true;
-        if (warp == 0) ok = issue(cur, 0, blk_lane, 0);
         int g = 0;  // ring position of the current item's first stage
         for (int k = 0; ok; ++k) {
             const int ntiles = (cur.ke - cur.kb + kKeys - 1) / kKeys;
-            const int idx_n = ring[(k + 1) & 3];
-            const bool has_next = idx_n < n_items;
-            int a_next = 0;
-            if (warp == 0 && lane == 0) a_next = atomicAdd(sched, 1);  // the item after next
+            const int spub = ntiles > 2 ? 2 : ntiles - 1;  // the stage after which the next index is readable
+            int idx_n = n_items;
+            bool has_next = false;
             DecodeItem nit{};
-            if (has_next) nit = p.ditems[idx_n];
             SeqInfo nsi{};
             DtGeo nxt{};
             uint32_t qn[D / 16][2];
-            int blk_lane_n = 0;
 
             float o[D / 16][4];
 #pragma unroll
             for (int mt = 0; mt < D / 16; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
             float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
             const int nkeys = cur.ke - cur.kb;
-            bool nready = false;
             for (int i = 0; i < ntiles; ++i) {
                 const int gs = g + i;
                 const int st = gs % kStages;
-                // the next item: its sequence row after stage 0, its block ids
-                // and query from stage 2 on (or before its first stage is issued)
-                if (has_next && !nready && (i == 2 || i == ntiles - 1)) {
-                    if (i == 0) nsi = p.seqs[nit.seq];
-                    nxt = geo_of(nit, nsi);
-                    load_q<D>(p, nxt.t, head, g8, c, qn);
-                    if (warp == 0) blk_lane_n = load_blk_lane(p, nxt, lane);
-                    nready = true;
-                }
-                if (warp == 0) {
-                    if (i + 1 < ntiles) ok = issue(cur, i + 1, blk_lane, gs + 1);
-                    else if (has_next) ok = issue(nxt, 0, blk_lane_n, gs + 1);
-                    if (!ok) break;
-                }
                 if (!wait(FULL(st), (gs / kStages) & 1)) { ok = false; break; }
+                if (i == spub) {  // the producer published it before issuing this stage
+                    idx_n = *reinterpret_cast<volatile int *>(ring + ((k + 1) & 3));
+                    has_next = idx_n < n_items;
+                    if (has_next) nit = p.ditems[idx_n];
+                }
                 const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
                 const int nv = nkeys - i * kKeys;  // valid keys in this stage (>= 1)
                 const bool tail = nv < kKeys;
@@ -368,8 +320,13 @@ __global__ void __launch_bounds__(kThreads, 4)
                 if (tail) tc::fence_proxy_async_smem();  // order the zeroing before the next TMA write
                 __syncwarp();
                 tc::mbar_arrive_warp(EMPTY(st));
-                if (i == 0 && has_next && !nready) nsi = p.seqs[nit.seq];
-                if (i == 1) settle();  // the previous item's counter, now that its stores are done
+                // the next item: its sequence row after this stage, its query a
+                // stage later (at once for a short item)
+                if (has_next && i == spub) nsi = p.seqs[nit.seq];
+                if (has_next && i == (spub + 1 < ntiles ? spub + 1 : spub)) {
+                    nxt = geo_of(nit, nsi);
+                    load_q<D>(p, nxt.t, head, g8, c, qn);
+                }
             }
             if (!ok) break;
             l0 += __shfl_xor_sync(0xffffffffu, l0, 4);
@@ -380,7 +337,6 @@ __global__ void __launch_bounds__(kThreads, 4)
             l1 += __shfl_xor_sync(0xffffffffu, l1, 16);
             const float inv0 = 1.f / l0, inv1 = 1.f / l1;
             const int h0 = 2 * c, h1 = 2 * c + 1;  // this lane's query heads within the group
-            settle();  // (the previous item, if this one had a single stage)
             if (cur.ns == 1) {
 #pragma unroll
                 for (int mt = 0; mt < D / 16; ++mt) {
@@ -421,29 +377,11 @@ __global__ void __launch_bounds__(kThreads, 4)
                     if (h1 < G) p.part_lse[part * Hq + head * G + h1] = m1 + log2f(l1);
                 }
             }
-            merge_if_last();  // the previous item's merge, with this item's accumulators stored
-            if (cur.ns > 1) {
-                pend = true;
-                pend_t = cur.t;
-                pend_ns = cur.ns;
-                pend_base = cur.part_base;
-                pend_group = cur.group;
-            }
-            // publish the item after next, then step to the next item
-            if (warp == 0 && lane == 0) ring[(k + 2) & 3] = a_next;
-            __syncwarp();
-            tc::mbar_arrive_warp(ITEMDONE(k & 1));
-            if (!wait(ITEMDONE(k & 1), (k >> 1) & 1)) break;
             if (!has_next) break;
             g += ntiles;
             cur = nxt;
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) { qb[kk][0] = qn[kk][0]; qb[kk][1] = qn[kk][1]; }
-            blk_lane = blk_lane_n;
-        }
-        if (!*abort_flag) {
-            settle();
-            merge_if_last();
         }
     }
 
@@ -456,6 +394,47 @@ __global__ void __launch_bounds__(kThreads, 4)
             __threadfence();
         }
     }
+}
+
+// Merge of the key splits of one decode token: out = sum_s w_s O_s / sum_s w_s,
+// w_s = 2^(lse_s - max), lse = max + log2(sum w) (the log-sum-exp combination
+// of partial softmax results). One warp per (split sequence, query head);
+// lanes hold four d columns each.
+template <int D>
+__global__ void __launch_bounds__(256) decode_merge_kernel(const AttnParams p) {
+    const int wg = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    const int Hq = p.num_q_heads;
+    pdl_wait();  // the decode grid's partial results
+    if (wg >= p.num_mgroups * Hq) return;
+    const MergeGroup mg = p.mgroups[wg / Hq];
+    const int h = wg % Hq;
+    const int ns = mg.num_splits, base = mg.part_base;
+    float M = -INFINITY;
+    for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, p.part_lse[static_cast<int64_t>(base + sp) * Hq + h]);
+#pragma unroll
+    for (int o2 = 16; o2 > 0; o2 >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o2));
+    float L = 0.f;
+    for (int sp = lane; sp < ns; sp += 32) L += fast_exp2(p.part_lse[static_cast<int64_t>(base + sp) * Hq + h] - M);
+#pragma unroll
+    for (int o2 = 16; o2 > 0; o2 >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o2);
+    if (lane < D / 4) {
+        const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+        for (int sp = 0; sp < ns; ++sp) {
+            const int64_t row = static_cast<int64_t>(base + sp) * Hq + h;
+            const float w = fast_exp2(p.part_lse[row] - M);
+            const float4 v = po[row * (D / 4) + lane];
+            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+        }
+        const float il = 1.f / L;
+        uint2 pk;
+        pk.x = pack_bf16x2(acc.x * il, acc.y * il);
+        pk.y = pack_bf16x2(acc.z * il, acc.w * il);
+        *reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.out) + (static_cast<int64_t>(mg.token) * Hq + h) * D +
+                                   lane * 4) = pk;
+    }
+    if (lane == 0) p.lse[static_cast<int64_t>(mg.token) * Hq + h] = (M + log2f(L)) * kLn2;
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -506,8 +485,7 @@ int launch_dt(const AttnParams &p, cudaStream_t st, int max_ctas) {
     FNPU_CUDA_TRY(cudaFuncSetAttribute(decode_tma_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                        cudaSharedmemCarveoutMaxShared));
     const int grid = p.num_ditems < max_ctas ? p.num_ditems : max_ctas;
-    decode_tma_kernel<D><<<grid, kThreads, Cfg::kSmemBytes, st>>>(p, maps);
-    FNPU_CUDA_TRY(cudaGetLastError());
+    FNPU_CUDA_TRY(launch_ex(decode_tma_kernel<D>, grid, kThreads, Cfg::kSmemBytes, st, false, nullptr, p, maps));
     return FNPU_OK;
 }
 
@@ -520,11 +498,19 @@ bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size)
 int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas) {
     if (p.num_ditems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int rc = FNPU_EUNSUPPORTED;
     switch (p.head_dim_qk) {
-        case 64: return launch_dt<64>(p, st, max_ctas);
-        case 128: return launch_dt<128>(p, st, max_ctas);
-        default: return FNPU_EUNSUPPORTED;
+        case 64: rc = launch_dt<64>(p, st, max_ctas); break;
+        case 128: rc = launch_dt<128>(p, st, max_ctas); break;
+        default: break;
     }
+    if (rc != FNPU_OK || p.num_mgroups == 0) return rc;
+    const int blocks = (p.num_mgroups * p.num_q_heads + 7) / 8;
+    // a dependent launch: its CTAs take the SMs that decode CTAs leave and
+    // wait there for the decode grid's writes
+    FNPU_CUDA_TRY(launch_ex(p.head_dim_qk == 64 ? decode_merge_kernel<64> : decode_merge_kernel<128>, blocks, 256, 0,
+                            st, true, nullptr, p));
+    return FNPU_OK;
 }
 
 }  // namespace fnpu

@@ -31,7 +31,9 @@ struct fnpu_plan {
     bool use_dt = false;
     bool use_mla = false;  // latent attention: one work list for both phases
     int32_t num_mitems = 0;
-    fnpu::MlaItem *d_mitems = nullptr;  // decode on the TMA-fed persistent kernel (items cover all kv heads)
+    fnpu::MlaItem *d_mitems = nullptr;
+    int32_t num_mgroups = 0;  // split decode tokens merged by the merge kernel
+    fnpu::MergeGroup *d_mgroups = nullptr;  // decode on the TMA-fed persistent kernel (items cover all kv heads)
     int32_t num_ditems = 0, num_pitems = 0, num_groups = 0, num_parts = 0;
     void *d_ws = nullptr;
     size_t ws_bytes = 0;
@@ -49,12 +51,12 @@ struct fnpu_plan {
     float *d_ppart_o = nullptr;
     int32_t num_pparts = 0, num_pgroups = 0;
     // co-location (Sec. 3.4): prefill CTAs on pre_ctas SMs and decode CTAs on
-    // the others, launched together on two library streams forked from and
-    // joined back into the caller's stream
+    // the others, launched on two library streams forked from and joined back
+    // into the caller's stream; e_started fires once all prefill CTAs began
     bool coloc = false;
     int32_t pre_ctas = 0;
     cudaStream_t s_pre = nullptr, s_dec = nullptr;
-    cudaEvent_t e_fork = nullptr, e_pre = nullptr, e_dec = nullptr;
+    cudaEvent_t e_fork = nullptr, e_started = nullptr, e_pre = nullptr, e_dec = nullptr;
 };
 
 namespace fnpu {
@@ -74,11 +76,12 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 void destroy_sync_objects(fnpu_plan *pl) {
     if (pl->s_pre) cudaStreamDestroy(pl->s_pre);
     if (pl->s_dec) cudaStreamDestroy(pl->s_dec);
+    if (pl->e_started) cudaEventDestroy(pl->e_started);
+    if (pl->e_dec) cudaEventDestroy(pl->e_dec);
     if (pl->e_fork) cudaEventDestroy(pl->e_fork);
     if (pl->e_pre) cudaEventDestroy(pl->e_pre);
-    if (pl->e_dec) cudaEventDestroy(pl->e_dec);
     pl->s_pre = pl->s_dec = nullptr;
-    pl->e_fork = pl->e_pre = pl->e_dec = nullptr;
+    pl->e_fork = pl->e_started = pl->e_pre = pl->e_dec = nullptr;
 }
 
 // Modelled rates of the two phases (measured on the co-located Qwen2.5-7B
@@ -342,16 +345,20 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     std::vector<PrefillItem> pitems;
     std::vector<std::pair<int64_t, int32_t>> pcost;  // (cost, index) for LPT order
     std::vector<TcUnit> tc_units;
+    std::vector<MergeGroup> mgroups;
 
-    // decode split length: about 3 waves of 2 CTAs per SM over the decode work
-    // (a TMA decode item streams every kv head of its keys)
+    // decode split length: the TMA decode CTAs (three per SM) share the
+    // bandwidth evenly, so the step lasts as long as the CTA with the most
+    // bytes; about four items per CTA keep that close to the mean (a TMA
+    // decode item streams every kv head of its keys). The per-head kernel
+    // aims at about 3 waves of 2 CTAs per SM.
     int64_t dec_keys = 0;
     for (int32_t s = 0; s < num_seqs; ++s)
         if (phase[s] == 1)
             dec_keys += static_cast<int64_t>(context_len[s]) * (pl->use_dt ? 1 : desc->num_kv_heads);
     int32_t split = o.decode_split_keys;
     if (split == 0) {
-        const int64_t target = 6LL * sms;
+        const int64_t target = (pl->use_dt ? 12LL : 6LL) * sms;
         int64_t sk = (dec_keys + target - 1) / std::max<int64_t>(target, 1);
         sk = (sk + 63) / 64 * 64;
         split = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(sk, pl->use_dt ? 128 : 256), 4096));
@@ -397,19 +404,18 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 }
             }
         } else if (phase[s] == 1 && pl->use_dt) {
-            // items over all kv heads; one merge counter per (sequence, kv head).
-            // At most 16 splits per sequence: the last split merges them, with
-            // one memory round trip per two splits, and a long sequence's merge
-            // would otherwise end the step late
-            const int32_t sk = std::max(split, (c + 16 * 64 - 1) / (16 * 64) * 64);
+            // items over all kv heads; a split sequence is merged by the merge
+            // kernel (at most 256 splits: its scratch grows with them)
+            const int32_t sk = std::max(split, (c + 256 * 64 - 1) / (256 * 64) * 64);
             const int32_t ns = (c + sk - 1) / sk;
-            const int32_t grp = groups;
-            groups += desc->num_kv_heads;
             const int32_t base = ns > 1 ? parts : 0;
-            if (ns > 1) parts += ns;
+            if (ns > 1) {
+                mgroups.push_back(MergeGroup{qs, ns, parts, 0});
+                parts += ns;
+            }
             for (int32_t sp = 0; sp < ns; ++sp) {
                 const int32_t kb = sp * sk, ke = std::min(c, kb + sk);
-                ditems.push_back(DecodeItem{s, 0, kb, ke, sp, ns, base, grp / desc->num_kv_heads});
+                ditems.push_back(DecodeItem{s, 0, kb, ke, sp, ns, base, 0});
             }
         } else if (phase[s] == 1) {
             const int32_t ns = (c + split - 1) / split;
@@ -500,6 +506,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         return (a.key_end - a.key_begin) > (b.key_end - b.key_begin);
     });
     pl->num_mitems = static_cast<int32_t>(mitems.size());
+    pl->num_mgroups = static_cast<int32_t>(mgroups.size());
     pl->num_ditems = static_cast<int32_t>(ditems.size());
     pl->num_pitems = static_cast<int32_t>(pordered.size());
     pl->num_groups = groups;
@@ -512,6 +519,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
             cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess ||
             cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess ||
             cudaEventCreateWithFlags(&pl->e_fork, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pl->e_started, cudaEventDisableTiming) != cudaSuccess ||
             cudaEventCreateWithFlags(&pl->e_pre, cudaEventDisableTiming) != cudaSuccess ||
             cudaEventCreateWithFlags(&pl->e_dec, cudaEventDisableTiming) != cudaSuccess) {
             cudaGetLastError();
@@ -527,6 +535,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_bt = off; off = align_up(off + sizeof(int32_t) * static_cast<size_t>(std::max(num_seqs, 1)) * width, 256);
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
     const size_t o_mi = off; off = align_up(off + sizeof(MlaItem) * std::max<size_t>(mitems.size(), 1), 256);
+    const size_t o_mg = off; off = align_up(off + sizeof(MergeGroup) * std::max<size_t>(mgroups.size(), 1), 256);
     const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
     const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
@@ -562,6 +571,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                sizeof(int32_t) * static_cast<size_t>((context_len[s] + bs - 1) / bs));
     if (!ditems.empty()) memcpy(h + o_di, ditems.data(), sizeof(DecodeItem) * ditems.size());
     if (!mitems.empty()) memcpy(h + o_mi, mitems.data(), sizeof(MlaItem) * mitems.size());
+    if (!mgroups.empty()) memcpy(h + o_mg, mgroups.data(), sizeof(MergeGroup) * mgroups.size());
     if (!pordered.empty()) memcpy(h + o_pi, pordered.data(), sizeof(PrefillItem) * pordered.size());
 
     uint8_t *d = static_cast<uint8_t *>(pl->d_ws);
@@ -569,6 +579,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->d_bt = reinterpret_cast<int32_t *>(d + o_bt);
     pl->d_ditems = reinterpret_cast<DecodeItem *>(d + o_di);
     pl->d_mitems = reinterpret_cast<MlaItem *>(d + o_mi);
+    pl->d_mgroups = reinterpret_cast<MergeGroup *>(d + o_mg);
     pl->d_pitems = reinterpret_cast<PrefillItem *>(d + o_pi);
     pl->d_counters = reinterpret_cast<int32_t *>(d + o_cnt);
     pl->d_err = reinterpret_cast<int32_t *>(d + o_err);
@@ -624,6 +635,8 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.scale_log2 = pl->scale * 1.4426950408889634f;
     p.ditems = pl->d_ditems;
     p.mitems = pl->d_mitems;
+    p.mgroups = pl->d_mgroups;
+    p.num_mgroups = pl->num_mgroups;
     p.num_mitems = pl->num_mitems;
     p.num_ditems = pl->num_ditems;
     p.part_o = pl->d_part_o;
@@ -641,16 +654,21 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     if (pl->coloc) {
         // both phases at once: pre_ctas persistent prefill CTAs (one per SM,
         // the tensor pipe; a decode CTA does not fit beside one) and decode
-        // CTAs on the other SMs (HBM). The prefill stream has the higher
-        // priority, so its CTAs are placed first; decode CTAs beyond the
-        // free SMs start on the SMs that the prefill leaves as its queue
-        // runs dry.
+        // CTAs on the other SMs (HBM). The decode stream waits for the event
+        // that fires once every prefill CTA has begun, so the decode grid
+        // only takes the SMs left over: with both grids pending at once the
+        // hardware may place either first, and stream priority alone does
+        // not settle it. Decode CTAs beyond the free SMs start on the SMs
+        // that the prefill leaves as its queue runs dry; the decode merge
+        // follows the decode grid on its stream, beside the prefill.
         cudaStream_t s = static_cast<cudaStream_t>(stream);
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
         FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
-        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
-        int rc = launch_prefill_tc(p, pl->s_pre, pl->pre_ctas);
-        if (rc == FNPU_OK) rc = launch_decode_tma(p, pl->s_dec, 3 * pl->num_sms);
+        int rc = launch_prefill_tc(p, pl->s_pre, pl->pre_ctas, pl->e_started);
+        if (rc == FNPU_OK) {
+            FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_started, 0));
+            rc = launch_decode_tma(p, pl->s_dec, 3 * pl->num_sms);
+        }
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
         FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_pre, 0));
@@ -698,7 +716,8 @@ int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_
     // latent attention has one work list for both phases, reported as prefill items
     if (prefill_items) *prefill_items = pl->num_pitems + pl->num_mitems;
     if (decode_items) *decode_items = pl->num_ditems;
-    if (launches_per_run) *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0);
+    if (launches_per_run)
+        *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0) + (pl->num_mgroups > 0);
     if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_bytes);
     return FNPU_OK;
 }

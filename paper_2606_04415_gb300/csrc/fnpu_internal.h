@@ -45,6 +45,13 @@ struct MlaItem {
 };
 static_assert(sizeof(MlaItem) == 48, "MlaItem layout");
 
+// The key splits of one decode token, merged by a separate kernel (TMA
+// decode path): partial rows part_base .. part_base + num_splits - 1.
+struct MergeGroup {
+    int32_t token, num_splits, part_base, pad;
+};
+static_assert(sizeof(MergeGroup) == 16, "MergeGroup layout");
+
 // Per-sequence metadata on the device.
 struct SeqInfo {
     int32_t q_start;  // first query token of the sequence in q/out/lse
@@ -74,7 +81,9 @@ struct AttnParams {
     int32_t num_ditems;
     float *part_o;          // fp32 [num_parts, group, dv]
     float *part_lse;        // fp32 [num_parts, group] (log2 domain)
-    int32_t *counters;      // [num_groups], zero between runs
+    int32_t *counters;      // [num_groups], zero between runs (per-head decode kernel)
+    const MergeGroup *mgroups;  // TMA decode path: split tokens to merge after the decode kernel
+    int32_t num_mgroups;
     // prefill
     const PrefillItem *pitems;
     int32_t num_pitems;
@@ -108,7 +117,8 @@ int launch_prefill_mma(const AttnParams &p, void *stream);
 int launch_mla(const AttnParams &p, void *stream);
 bool mla_supported(int d_qk, int d_v, int hq, int hkv);
 int mla_heads_per_item();
-int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas);
+// started (a cudaEvent_t, may be null): recorded once every CTA has begun
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started = nullptr);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
 int prefill_tc_rows_per_item(int group);
 int prefill_tc_keys_per_tile();

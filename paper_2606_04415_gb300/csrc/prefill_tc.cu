@@ -660,7 +660,7 @@ bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, in
 }
 
 template <int D>
-int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas) {
+int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t started) {
     using Cfg = TcCfg<D>;
     TcMaps maps;
     if (!encode_cache_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
@@ -672,8 +672,7 @@ int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas) {
     FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                        cudaSharedmemCarveoutMaxShared));
     const int grid = p.num_pitems < max_ctas ? p.num_pitems : max_ctas;
-    prefill_tc_kernel<D><<<grid, kThreads, Cfg::kSmemBytes, st>>>(p, maps);
-    FNPU_CUDA_TRY(cudaGetLastError());
+    FNPU_CUDA_TRY(launch_ex(prefill_tc_kernel<D>, grid, kThreads, Cfg::kSmemBytes, st, false, started, p, maps));
     return FNPU_OK;
 }
 
@@ -690,12 +689,12 @@ int prefill_tc_rows_per_item(int group) { return 2 * (kRows / group); }
 // keys per K/V tile (the unit of the planner's key splits)
 int prefill_tc_keys_per_tile() { return kKeys; }
 
-int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas) {
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started) {
     if (p.num_pitems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     switch (p.head_dim_qk) {
-        case 64: return launch_tc<64>(p, st, max_ctas);
-        case 128: return launch_tc<128>(p, st, max_ctas);
+        case 64: return launch_tc<64>(p, st, max_ctas, static_cast<cudaEvent_t>(started));
+        case 128: return launch_tc<128>(p, st, max_ctas, static_cast<cudaEvent_t>(started));
         default: return FNPU_EUNSUPPORTED;
     }
 }
