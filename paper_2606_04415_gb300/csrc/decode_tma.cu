@@ -398,35 +398,59 @@ __global__ void __launch_bounds__(kThreads, 3)
 
 // Merge of the key splits of one decode token: out = sum_s w_s O_s / sum_s w_s,
 // w_s = 2^(lse_s - max), lse = max + log2(sum w) (the log-sum-exp combination
-// of partial softmax results). One warp per (split sequence, query head);
-// lanes hold four d columns each.
+// of partial softmax results). One warp per (split sequence, query head),
+// lanes holding four d columns each. The splits go in chunks of 32: a chunk's
+// log-sum-exps take one load per lane, its weights reach the other lanes by
+// shuffle, and a running maximum rescales what earlier chunks summed; the
+// partial rows stream 16 at a time, so a token of up to 32 splits costs two
+// memory round trips after the decode grid.
+constexpr int kMergeWarps = 4;
+
 template <int D>
-__global__ void __launch_bounds__(256) decode_merge_kernel(const AttnParams p) {
-    const int wg = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+__global__ void __launch_bounds__(32 * kMergeWarps) decode_merge_kernel(const AttnParams p) {
+    const int wg = blockIdx.x * kMergeWarps + (threadIdx.x >> 5), lane = threadIdx.x & 31;
     const int Hq = p.num_q_heads;
     pdl_wait();  // the decode grid's partial results
     if (wg >= p.num_mgroups * Hq) return;
     const MergeGroup mg = p.mgroups[wg / Hq];
     const int h = wg % Hq;
     const int ns = mg.num_splits, base = mg.part_base;
-    float M = -INFINITY;
-    for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, p.part_lse[static_cast<int64_t>(base + sp) * Hq + h]);
+    const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
+    const bool col = lane < D / 4;
+    float M = -INFINITY, L = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c0 = 0; c0 < ns; c0 += 32) {
+        const int nc = ns - c0 < 32 ? ns - c0 : 32;
+        const float my = lane < nc ? __ldcg(p.part_lse + static_cast<int64_t>(base + c0 + lane) * Hq + h) : -INFINITY;
+        float cm = my;
 #pragma unroll
-    for (int o2 = 16; o2 > 0; o2 >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o2));
-    float L = 0.f;
-    for (int sp = lane; sp < ns; sp += 32) L += fast_exp2(p.part_lse[static_cast<int64_t>(base + sp) * Hq + h] - M);
+        for (int o2 = 16; o2 > 0; o2 >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, o2));
+        const float Mn = fmaxf(M, cm);
+        const float a = fast_exp2(M - Mn);  // 0 for the first chunk (M = -inf)
+        const float w = fast_exp2(my - Mn);  // this lane's split weight, 0 past the chunk
+        float cl = w;
 #pragma unroll
-    for (int o2 = 16; o2 > 0; o2 >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o2);
-    if (lane < D / 4) {
-        const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-        for (int sp = 0; sp < ns; ++sp) {
-            const int64_t row = static_cast<int64_t>(base + sp) * Hq + h;
-            const float w = fast_exp2(p.part_lse[row] - M);
-            const float4 v = po[row * (D / 4) + lane];
-            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+        for (int o2 = 16; o2 > 0; o2 >>= 1) cl += __shfl_xor_sync(0xffffffffu, cl, o2);
+        L = L * a + cl;
+        acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
+        M = Mn;
+        // lanes past d (D = 64) read a duplicate column and drop it
+        const float4 *row = po + (static_cast<int64_t>(base + c0) * Hq + h) * (D / 4) + (lane & (D / 4 - 1));
+        for (int j0 = 0; j0 < nc; j0 += 16) {
+            float4 v[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u)
+                if (j0 + u < nc) v[u] = __ldcg(row + static_cast<int64_t>(j0 + u) * Hq * (D / 4));
+#pragma unroll
+            for (int u = 0; u < 16; ++u) {
+                if (j0 + u < nc) {
+                    const float wj = __shfl_sync(0xffffffffu, w, j0 + u);
+                    acc.x += wj * v[u].x; acc.y += wj * v[u].y; acc.z += wj * v[u].z; acc.w += wj * v[u].w;
+                }
+            }
         }
+    }
+    if (col) {
         const float il = 1.f / L;
         uint2 pk;
         pk.x = pack_bf16x2(acc.x * il, acc.y * il);
@@ -505,11 +529,11 @@ int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas) {
         default: break;
     }
     if (rc != FNPU_OK || p.num_mgroups == 0) return rc;
-    const int blocks = (p.num_mgroups * p.num_q_heads + 7) / 8;
+    const int blocks = (p.num_mgroups * p.num_q_heads + kMergeWarps - 1) / kMergeWarps;
     // a dependent launch: its CTAs take the SMs that decode CTAs leave and
     // wait there for the decode grid's writes
-    FNPU_CUDA_TRY(launch_ex(p.head_dim_qk == 64 ? decode_merge_kernel<64> : decode_merge_kernel<128>, blocks, 256, 0,
-                            st, true, nullptr, p));
+    FNPU_CUDA_TRY(launch_ex(p.head_dim_qk == 64 ? decode_merge_kernel<64> : decode_merge_kernel<128>, blocks,
+                            32 * kMergeWarps, 0, st, true, nullptr, p));
     return FNPU_OK;
 }
 
