@@ -396,29 +396,33 @@ __global__ void __launch_bounds__(kThreads, 3)
     }
 }
 
-// Merge of the key splits of one decode token: out = sum_s w_s O_s / sum_s w_s,
+// Merge of the key splits of one query token: out = sum_s w_s O_s / sum_s w_s,
 // w_s = 2^(lse_s - max), lse = max + log2(sum w) (the log-sum-exp combination
-// of partial softmax results). One warp per (split sequence, query head),
-// lanes holding four d columns each. The splits go in chunks of 32: a chunk's
-// log-sum-exps take one load per lane, its weights reach the other lanes by
-// shuffle, and a running maximum rescales what earlier chunks summed; the
-// partial rows stream 16 at a time, so a token of up to 32 splits costs two
-// memory round trips after the decode grid.
+// of partial softmax results). One warp per (split token, query head), lanes
+// holding float4 columns lane, lane + 32, ... of the row. The splits go in
+// chunks of 32: a chunk's log-sum-exps take one load per lane, its weights
+// reach the other lanes by shuffle, and a running maximum rescales what
+// earlier chunks summed; the partial rows stream with 16 float4 per lane in
+// flight, so a token of up to 32 splits costs a few memory round trips.
 constexpr int kMergeWarps = 4;
 
 template <int D>
-__global__ void __launch_bounds__(32 * kMergeWarps) decode_merge_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(32 * kMergeWarps) split_merge_kernel(const AttnParams p) {
+    constexpr int kV = D / 4;                 // float4 per row
+    constexpr int kC = (kV + 31) / 32;        // float4 columns per lane
+    constexpr int kB = 16 / kC;               // partial rows in flight
     const int wg = blockIdx.x * kMergeWarps + (threadIdx.x >> 5), lane = threadIdx.x & 31;
     const int Hq = p.num_q_heads;
-    pdl_wait();  // the decode grid's partial results
+    pdl_wait();  // the partial results of the grid before
     if (wg >= p.num_mgroups * Hq) return;
     const MergeGroup mg = p.mgroups[wg / Hq];
     const int h = wg % Hq;
     const int ns = mg.num_splits, base = mg.part_base;
     const float4 *po = reinterpret_cast<const float4 *>(p.part_o);
-    const bool col = lane < D / 4;
     float M = -INFINITY, L = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4 acc[kC];
+#pragma unroll
+    for (int c = 0; c < kC; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int c0 = 0; c0 < ns; c0 += 32) {
         const int nc = ns - c0 < 32 ? ns - c0 : 32;
         const float my = lane < nc ? __ldcg(p.part_lse + static_cast<int64_t>(base + c0 + lane) * Hq + h) : -INFINITY;
@@ -432,31 +436,44 @@ __global__ void __launch_bounds__(32 * kMergeWarps) decode_merge_kernel(const At
 #pragma unroll
         for (int o2 = 16; o2 > 0; o2 >>= 1) cl += __shfl_xor_sync(0xffffffffu, cl, o2);
         L = L * a + cl;
-        acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
+#pragma unroll
+        for (int c = 0; c < kC; ++c) {
+            acc[c].x *= a; acc[c].y *= a; acc[c].z *= a; acc[c].w *= a;
+        }
         M = Mn;
-        // lanes past d (D = 64) read a duplicate column and drop it
-        const float4 *row = po + (static_cast<int64_t>(base + c0) * Hq + h) * (D / 4) + (lane & (D / 4 - 1));
-        for (int j0 = 0; j0 < nc; j0 += 16) {
-            float4 v[16];
+        // lanes past the row (D = 64) read a duplicate column and drop it
+        const float4 *row = po + (static_cast<int64_t>(base + c0) * Hq + h) * kV + (lane & (kV < 32 ? kV - 1 : 31));
+        for (int j0 = 0; j0 < nc; j0 += kB) {
+            float4 v[kB][kC];
 #pragma unroll
-            for (int u = 0; u < 16; ++u)
-                if (j0 + u < nc) v[u] = __ldcg(row + static_cast<int64_t>(j0 + u) * Hq * (D / 4));
+            for (int u = 0; u < kB; ++u)
+                if (j0 + u < nc) {
 #pragma unroll
-            for (int u = 0; u < 16; ++u) {
+                    for (int c = 0; c < kC; ++c) v[u][c] = __ldcg(row + static_cast<int64_t>(j0 + u) * Hq * kV + 32 * c);
+                }
+#pragma unroll
+            for (int u = 0; u < kB; ++u) {
                 if (j0 + u < nc) {
                     const float wj = __shfl_sync(0xffffffffu, w, j0 + u);
-                    acc.x += wj * v[u].x; acc.y += wj * v[u].y; acc.z += wj * v[u].z; acc.w += wj * v[u].w;
+#pragma unroll
+                    for (int c = 0; c < kC; ++c) {
+                        acc[c].x += wj * v[u][c].x; acc[c].y += wj * v[u][c].y;
+                        acc[c].z += wj * v[u][c].z; acc[c].w += wj * v[u][c].w;
+                    }
                 }
             }
         }
     }
-    if (col) {
-        const float il = 1.f / L;
-        uint2 pk;
-        pk.x = pack_bf16x2(acc.x * il, acc.y * il);
-        pk.y = pack_bf16x2(acc.z * il, acc.w * il);
-        *reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.out) + (static_cast<int64_t>(mg.token) * Hq + h) * D +
-                                   lane * 4) = pk;
+    const float il = 1.f / L;
+    __nv_bfloat16 *orow = static_cast<__nv_bfloat16 *>(p.out) + (static_cast<int64_t>(mg.token) * Hq + h) * D;
+#pragma unroll
+    for (int c = 0; c < kC; ++c) {
+        if (32 * c + lane < kV) {
+            uint2 pk;
+            pk.x = pack_bf16x2(acc[c].x * il, acc[c].y * il);
+            pk.y = pack_bf16x2(acc[c].z * il, acc[c].w * il);
+            *reinterpret_cast<uint2 *>(orow + (32 * c + lane) * 4) = pk;
+        }
     }
     if (lane == 0) p.lse[static_cast<int64_t>(mg.token) * Hq + h] = (M + log2f(L)) * kLn2;
 }
@@ -528,12 +545,24 @@ int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas) {
         case 128: rc = launch_dt<128>(p, st, max_ctas); break;
         default: break;
     }
-    if (rc != FNPU_OK || p.num_mgroups == 0) return rc;
+    if (rc != FNPU_OK) return rc;
+    return launch_split_merge(p, stream);
+}
+
+int launch_split_merge(const AttnParams &p, void *stream) {
+    if (p.num_mgroups == 0) return FNPU_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int blocks = (p.num_mgroups * p.num_q_heads + kMergeWarps - 1) / kMergeWarps;
-    // a dependent launch: its CTAs take the SMs that decode CTAs leave and
-    // wait there for the decode grid's writes
-    FNPU_CUDA_TRY(launch_ex(p.head_dim_qk == 64 ? decode_merge_kernel<64> : decode_merge_kernel<128>, blocks,
-                            32 * kMergeWarps, 0, st, true, nullptr, p));
+    void (*kernel)(AttnParams) = nullptr;
+    switch (p.head_dim_v) {
+        case 64: kernel = split_merge_kernel<64>; break;
+        case 128: kernel = split_merge_kernel<128>; break;
+        case 512: kernel = split_merge_kernel<512>; break;
+        default: return FNPU_EUNSUPPORTED;
+    }
+    // a dependent launch: its CTAs take the SMs that the CTAs of the grid
+    // before leave and wait there for that grid's writes
+    FNPU_CUDA_TRY(launch_ex(kernel, blocks, 32 * kMergeWarps, 0, st, true, nullptr, p));
     return FNPU_OK;
 }
 

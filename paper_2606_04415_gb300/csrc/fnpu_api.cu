@@ -30,6 +30,7 @@ struct fnpu_plan {
     bool use_tc = false;
     bool use_dt = false;
     bool use_mla = false;  // latent attention: one work list for both phases
+    bool use_mla_tc = false;  // ... on the tcgen05 kernel (items of 128 heads and one d_v half)
     int32_t num_mitems = 0;
     fnpu::MlaItem *d_mitems = nullptr;
     int32_t num_mgroups = 0;  // split decode tokens merged by the merge kernel
@@ -333,6 +334,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->num_sms = sms;
     pl->flags = o.flags;
     pl->use_mla = desc->v_in_k_latent != 0;
+    pl->use_mla_tc = pl->use_mla && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
+                     mla_tc_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_q_heads, desc->num_kv_heads, bs);
     pl->use_dt = !pl->use_mla && decode_tma_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_kv_heads,
                                                       desc->num_q_heads / desc->num_kv_heads, bs);
     pl->use_tc = !pl->use_mla && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
@@ -369,7 +372,19 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     // that about three CTAs per SM share the work; longest first
     std::vector<MlaItem> mitems;
     int32_t mla_split = 0;
-    if (pl->use_mla) {
+    int32_t mla_split_tiles = 0;
+    if (pl->use_mla_tc) {
+        // two CTAs (d_v halves) per piece, 64-key tiles; a token is cut only
+        // when it alone would exceed half of an SM's mean share of the tiles
+        // (then pieces of whole tiles, at least 16 of them)
+        const int32_t kt = mla_tc_keys_per_tile();
+        int64_t tiles = 0;
+        for (int32_t s = 0; s < num_seqs; ++s)
+            for (int32_t i = 0; i < query_len[s]; ++i)
+                tiles += 2 * ((context_len[s] - query_len[s] + i + 1 + kt - 1) / kt);
+        const int64_t half_mean = (tiles + 2LL * sms - 1) / (2LL * sms);
+        mla_split_tiles = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(half_mean, 16), 1 << 20));
+    } else if (pl->use_mla) {
         int64_t rows_keys = 0;
         for (int32_t s = 0; s < num_seqs; ++s) {
             const int64_t q = query_len[s], p0 = context_len[s] - query_len[s];
@@ -386,7 +401,24 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     for (int32_t s = 0; s < num_seqs; ++s) {
         seqs[s] = SeqInfo{qs, query_len[s], context_len[s], s};
         const int32_t q = query_len[s], c = context_len[s];
-        if (pl->use_mla) {
+        if (pl->use_mla_tc) {
+            const int32_t kt = mla_tc_keys_per_tile();
+            for (int32_t i = 0; i < q; ++i) {
+                const int32_t keys = c - q + i + 1;
+                const int32_t nt = (keys + kt - 1) / kt;
+                const int32_t ns = (nt + mla_split_tiles - 1) / mla_split_tiles;
+                const int32_t per = (nt + ns - 1) / ns;  // tiles per piece
+                const int32_t base = ns > 1 ? parts : 0;
+                if (ns > 1) {
+                    mgroups.push_back(MergeGroup{qs + i, ns, parts, 0});
+                    parts += ns;
+                }
+                for (int32_t sp = 0; sp < ns; ++sp)
+                    for (int32_t h = 0; h < 2; ++h)  // the two d_v halves, next to each other
+                        mitems.push_back(MlaItem{s, i, h, sp * per * kt, std::min(keys, (sp + 1) * per * kt), sp, ns,
+                                                 base, 0, 0, 0, 0});
+            }
+        } else if (pl->use_mla) {
             const int32_t nhb = desc->num_q_heads / mla_heads_per_item();
             for (int32_t i = 0; i < q; ++i) {
                 const int32_t keys = c - q + i + 1;
@@ -542,7 +574,9 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
     const size_t meta_bytes = off;
     // query heads per partial
-    const int32_t part_rows = pl->use_mla ? mla_heads_per_item() : (pl->use_dt ? desc->num_q_heads : G);
+    const int32_t part_rows = pl->use_mla_tc ? desc->num_q_heads
+                              : pl->use_mla  ? mla_heads_per_item()
+                                             : (pl->use_dt ? desc->num_q_heads : G);
     const size_t o_plse = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows, 256);
     const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows * desc->head_dim_v, 256);
     const size_t o_pplse = off; off = align_up(off + sizeof(float) * 256 * static_cast<size_t>(std::max(pparts, 1)), 256);
@@ -650,7 +684,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
 
-    if (pl->use_mla) return launch_mla(p, stream);
+    if (pl->use_mla) return pl->use_mla_tc ? launch_mla_tc(p, stream) : launch_mla(p, stream);
     if (pl->coloc) {
         // both phases at once: pre_ctas persistent prefill CTAs (one per SM,
         // the tensor pipe; a decode CTA does not fit beside one) and decode

@@ -115,6 +115,12 @@ int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas);
 bool decode_tma_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_prefill_mma(const AttnParams &p, void *stream);
 int launch_mla(const AttnParams &p, void *stream);
+// tcgen05 latent attention: items are (token, d_v half, key range) of 128 heads
+int launch_mla_tc(const AttnParams &p, void *stream);
+bool mla_tc_supported(int d_qk, int d_v, int hq, int hkv, int block_size);
+int mla_tc_keys_per_tile();
+// log-sum-exp merge of the split tokens listed in p.mgroups (partials [part, Hq, dv])
+int launch_split_merge(const AttnParams &p, void *stream);
 bool mla_supported(int d_qk, int d_v, int hq, int hkv);
 int mla_heads_per_item();
 // started (a cudaEvent_t, may be null): recorded once every CTA has begun

@@ -306,11 +306,14 @@ def test_colocated_launch_matches_separate_launches(share):
     assert np.abs(a_out - b_out).max() <= O_TOL and np.abs(a_lse - b_lse).max() <= LSE_TOL
 
 
-@pytest.mark.parametrize("bs", [16, 64])
-def test_mla_small_mixed_batch_all_rows(bs):
+@pytest.mark.parametrize("flags", [0, NO_TC])
+@pytest.mark.parametrize("bs", [16, 32, 64])
+def test_mla_small_mixed_batch_all_rows(bs, flags):
     """Absorbed MLA (128 heads on one 576-wide latent, V = its first 512
     columns): prefill chunks with and without prefix, decodes long enough to
-    be split and merged, ragged lengths; every row against the oracle. The
+    be split and merged, ragged lengths (tiles past a sequence's last block,
+    pieces ending inside a block); every row against the oracle, on the
+    tcgen05 kernel (d_v halves, merge kernel) and on the mma.sync kernel. The
     latent KV append is bit-exact."""
     sh = W.Shape(128, 1, 576, 512, bs, True)
     ql = [7, 1, 1, 33, 1, 1]
@@ -318,7 +321,7 @@ def test_mla_small_mixed_batch_all_rows(bs):
     ph = [0, 1, 1, 0, 1, 1]
     rng = np.random.default_rng(500 + bs)
     batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_small")
-    st = _step(batch)
+    st = _step(batch, flags=flags)
     kc, _ = st.cache_bits()
     assert np.array_equal(kc, oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping))
     out, lse = st.results()
