@@ -40,7 +40,7 @@ import numpy as np
 
 BF16_CANARY = np.uint16(0x7FC1)  # a quiet NaN with a distinct payload
 
-CONFIG_NAMES = ("tiny", "qwen_decode", "qwen_prefill", "qwen_coloc", "mla_coloc")
+CONFIG_NAMES = ("tiny", "qwen_decode", "qwen_prefill", "qwen_coloc", "mla_coloc", "mla_coloc_small")
 
 
 @dataclasses.dataclass(frozen=True)
@@ -156,6 +156,14 @@ def draw_lengths(name: str, rng: np.random.Generator):
         q = [1024] + [1] * 256
         ctx = [1024] + dec.tolist()
         ph = [0] + [1] * 256
+    elif name == "mla_coloc_small":
+        # the MLA co-located mix at about a quarter of the size (for profiler
+        # captures, which replay a kernel many times): one 256-token prompt
+        # (no prefix) + 48 decodes, ctx ~ U[4096, 16384]
+        dec = rng.integers(4096, 16384, endpoint=True, size=48)
+        q = [256] + [1] * 48
+        ctx = [256] + dec.tolist()
+        ph = [0] + [1] * 48
     else:
         raise ValueError(f"unknown workload {name!r}")
     return (np.asarray(q, np.int32), np.asarray(ctx, np.int32), np.asarray(ph, np.uint8))
