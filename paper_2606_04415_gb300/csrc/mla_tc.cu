@@ -87,6 +87,17 @@ __global__ void __launch_bounds__(kThreads, 1) mla_tc_kernel(const AttnParams p,
         if (tid == 0) atomicOr(p.err, 2);
         return;
     }
+    // Q columns 192..575 of this head (softmax warps), loaded before the
+    // set-up so that their memory latency overlaps it: all 48 16-byte loads
+    // in flight at once
+    constexpr int kQtLoads = (kTmemCols - kColQ) * 4 / 16;  // 48
+    uint4 qv[kQtLoads];
+    if (warp < 4) {
+        const uint4 *qrow = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(p.q) +
+                                                            (tok * kRows + tid) * kDq + 64 * kQsChunks);
+#pragma unroll
+        for (int u = 0; u < kQtLoads; ++u) qv[u] = __ldg(qrow + u);
+    }
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(FULL(s), 1);
@@ -210,14 +221,12 @@ __global__ void __launch_bounds__(kThreads, 1) mla_tc_kernel(const AttnParams p,
         // Q columns 192..575 of this head, packed in bf16 pairs, into tensor
         // memory (the A operand of the TS steps of S)
         {
-            const uint4 *qrow = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(p.q) +
-                                                                (tok * kRows + r) * kDq + 64 * kQsChunks);
-#pragma unroll 1
+#pragma unroll
             for (int c = 0; c < (kTmemCols - kColQ) / 32; ++c) {
                 uint32_t v[32];
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
-                    const uint4 x = __ldg(qrow + c * 8 + u);
+                    const uint4 x = qv[c * 8 + u];
                     v[4 * u] = x.x; v[4 * u + 1] = x.y; v[4 * u + 2] = x.z; v[4 * u + 3] = x.w;
                 }
                 tc::tmem_st32(lane_addr + kColQ + 32 * c, v);

@@ -347,3 +347,43 @@ def test_mla_coloc_full_size_sampled_rows():
         q = int(batch.query_len[s])
         toks += [int(qs[s]) + r for r in sorted({0, 1, 63, 64, q - 1, int(rng.integers(0, q))})]
     _compare(batch, out, lse, tokens=np.asarray(sorted(set(toks)), np.int64))
+
+
+@pytest.mark.parametrize("heads", [64, 256])
+def test_mla_other_head_counts(heads):
+    """Latent attention with 64 or 256 query heads (the mma.sync kernel: the
+    tcgen05 one takes exactly 128 rows per token); a split decode and a
+    prefill chunk on a prefix; every row against the oracle."""
+    sh = W.Shape(heads, 1, 576, 512, 64, True)
+    ql, ctx, ph = [1, 20, 1], [2200, 20 + 70, 300], [1, 0, 1]
+    rng = np.random.default_rng(900 + heads)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_heads")
+    out, lse = _step(batch).results()
+    _compare(batch, out, lse)
+
+
+def test_mla_long_decode_many_pieces():
+    """One 40000-key latent decode beside a short one: the planner cuts it into
+    about 40 pieces of 16 tiles, so the d_v = 512 merge runs more than one
+    32-split chunk (running maximum across chunks)."""
+    sh = W.Shape(128, 1, 576, 512, 64, True)
+    ql, ctx, ph = [1, 1], [40000, 77], [1, 1]
+    rng = np.random.default_rng(910)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_long")
+    st = _step(batch)
+    assert st.plan.info()["prefill_items"] > 2 * 32
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_decode_long_token_many_splits():
+    """A lone 8192-key decode on the TMA decode kernel: 128-key items give it
+    64 splits, two 32-split chunks in the merge kernel."""
+    sh = W.SHAPES["qwen"]
+    ql, ctx, ph = [1, 1], [8192, 300], [1, 1]
+    rng = np.random.default_rng(920)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="long_decode")
+    st = _step(batch)
+    assert st.plan.info()["decode_items"] >= 64
+    out, lse = st.results()
+    _compare(batch, out, lse)
