@@ -478,7 +478,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 for (int32_t h = 0; h < desc->num_q_heads; ++h) {
                     pcost.emplace_back(static_cast<int64_t>(prefix) + r0 + rows,
                                        static_cast<int32_t>(pitems.size()));
-                    pitems.push_back(PrefillItem{s, h, r0, rows, 0, 0, 0, 1, 0, 0, 0, 0});
+                    pitems.push_back(PrefillItem{s, h, r0, rows, 0, 0, 0, 1, 0, 0, qs, prefix, c, s, 0, 0});
                 }
             }
         }
@@ -518,7 +518,9 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 const int32_t kb = split_bound(t.ntiles, n, j), ke = split_bound(t.ntiles, n, j + 1);
                 pcost.emplace_back(static_cast<int64_t>(ke - kb) + kTcItemCost + (n > 1 ? kTcMergeCost : 0),
                                    static_cast<int32_t>(pitems.size()));
-                pitems.push_back(PrefillItem{t.seq, t.kvh, t.r0, t.rows, kb, ke, j, n, base, grp, 0, 0});
+                pitems.push_back(PrefillItem{t.seq, t.kvh, t.r0, t.rows, kb, ke, j, n, base, grp,
+                                             seqs[t.seq].q_start, seqs[t.seq].ctx_len - seqs[t.seq].q_len,
+                                             seqs[t.seq].ctx_len, seqs[t.seq].bt_row, 0, 0});
             }
         }
     }

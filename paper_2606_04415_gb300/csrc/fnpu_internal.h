@@ -30,9 +30,11 @@ static_assert(sizeof(DecodeItem) == 32, "DecodeItem layout");
 struct PrefillItem {
     int32_t seq, head, row_begin, rows;
     int32_t kt_begin, kt_end, split, num_splits;
-    int32_t part_base, group, pad0, pad1;
+    int32_t part_base, group;
+    int32_t q_start, prefix, ctx_len, bt_row;  // the sequence's SeqInfo, so one load decodes an item
+    int32_t pad0, pad1;
 };
-static_assert(sizeof(PrefillItem) == 48, "PrefillItem layout");
+static_assert(sizeof(PrefillItem) == 64, "PrefillItem layout");
 
 // One latent-attention (MLA) work item: query heads [64 hb, 64 hb + 64) of
 // query row `row` of sequence `seq` (a prefill or a decode row alike) over

@@ -94,18 +94,17 @@ struct ItemGeom {
 };
 
 __device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
-    const PrefillItem it = p.pitems[idx];
-    const SeqInfo si = p.seqs[it.seq];
+    const PrefillItem it = p.pitems[idx];  // carries its sequence's fields: one load
     ItemGeom g;
     g.kvh = it.head;
     g.p0 = it.row_begin;
     g.rows = it.rows;
-    g.prefix = si.ctx_len - si.q_len;
-    g.ctx = si.ctx_len;
+    g.prefix = it.prefix;
+    g.ctx = it.ctx_len;
     g.kt0 = it.kt_begin;              // 128-key tiles [kt_begin, kt_end) of keys 0 .. last position
     g.ntiles = it.kt_end - it.kt_begin;
-    g.q_start = si.q_start;
-    g.bt_row = si.bt_row;
+    g.q_start = it.q_start;
+    g.bt_row = it.bt_row;
     g.ns = it.num_splits;
     g.split = it.split;
     g.pbase = it.part_base;
@@ -207,7 +206,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int slot = k & 1;
             int idx = 0;
             if (is_k) {
-                if (lane == 0) idx = atomicAdd(p.sched, 1);
+                // the first item of CTA b is item b (the queue hands the first
+                // gridDim.x items out in that order anyway); later ones come
+                // from the queue
+                if (lane == 0) idx = k == 0 ? static_cast<int>(blockIdx.x) : static_cast<int>(gridDim.x) + atomicAdd(p.sched, 1);
                 idx = __shfl_sync(0xffffffffu, idx, 0);
                 if (k >= 2 && !wait(ITEMEMPTY(slot), ((k >> 1) - 1) & 1)) break;
                 if (lane == 0) {
@@ -222,17 +224,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const ItemGeom it = item_geom(p, idx);
             const int ukvh = __shfl_sync(0xffffffffu, it.kvh, 0);
-            if (is_k) {  // both Q tiles, once the previous item's last S is done
-                if (k >= 1 && !wait(QEMPTY, (k - 1) & 1)) break;
+            // both Q tiles, once the previous item's last S is done (loading them
+            // after the item's first K tiles, with an L2 prefetch ahead, was
+            // measured slower)
+            const int q0 = __shfl_sync(0xffffffffu, it.q_start + it.p0, 0);
+            auto load_q = [&]() -> bool {
+                if (k >= 1 && !wait(QEMPTY, (k - 1) & 1)) return false;
                 tc::mbar_arrive_expect_tx_warp(QFULL, static_cast<uint32_t>(2 * (D / 64) * 64 * G * P * 2));
-                const int q0 = __shfl_sync(0xffffffffu, it.q_start + it.p0, 0);
 #pragma unroll
                 for (int w = 0; w < 2; ++w)
 #pragma unroll
                     for (int h = 0; h < D / 64; ++h)
                         tc::tma_load_3d_warp(s_base + Cfg::kQOff + w * Cfg::kQBytes + h * Cfg::kQHalf, &maps.q,
                                              QFULL, h * 64, ukvh * G, q0 + w * P);
-            }
+                return true;
+            };
             const int32_t *bt = p.block_table + static_cast<int64_t>(it.bt_row) * p.bt_stride;
             const int nblk_seq = (it.ctx + bs - 1) / bs;
             // block ids of the next tile, one per lane, loaded a tile ahead so
@@ -241,6 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int blk_next = (lane < per_tile && b00 + lane < nblk_seq) ? __ldg(bt + b00 + lane) : 0;
             bool ok = true;
             for (int i = 0; i < it.ntiles; ++i, ++g) {
+                if (is_k && i == 0 && !load_q()) { ok = false; break; }
                 const int st = g % nst;
                 const int blk_cur = blk_next;
                 const int jn = b00 + (i + 1) * per_tile + lane;
