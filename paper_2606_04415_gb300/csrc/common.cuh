@@ -142,6 +142,14 @@ cudaError_t launch_ex(void (*kernel)(Args...), int grid, int threads, size_t sme
     return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
+// One 32-byte global store (8 x 32 bits; the address is 32-byte aligned).
+__device__ __forceinline__ void st_global_v8(void *ptr, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                             uint32_t a4, uint32_t a5, uint32_t a6, uint32_t a7) {
+    asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};\n" ::"l"(ptr), "r"(a0), "r"(a1), "r"(a2),
+                 "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+                 : "memory");
+}
+
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 

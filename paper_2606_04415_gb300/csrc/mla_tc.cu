@@ -329,13 +329,13 @@ __global__ void __launch_bounds__(kThreads, 1) mla_tc_kernel(const AttnParams p,
                     tc::tmem_ld32(lane_addr + kColO + 32 * c, o);
                     tc::tmem_wait_ld();
 #pragma unroll
-                    for (int x = 0; x < 4; ++x) {
-                        uint4 v;
-                        v.x = pack_bf16x2(__uint_as_float(o[8 * x + 0]) * inv, __uint_as_float(o[8 * x + 1]) * inv);
-                        v.y = pack_bf16x2(__uint_as_float(o[8 * x + 2]) * inv, __uint_as_float(o[8 * x + 3]) * inv);
-                        v.z = pack_bf16x2(__uint_as_float(o[8 * x + 4]) * inv, __uint_as_float(o[8 * x + 5]) * inv);
-                        v.w = pack_bf16x2(__uint_as_float(o[8 * x + 6]) * inv, __uint_as_float(o[8 * x + 7]) * inv);
-                        orow[c * 4 + x] = v;
+                    for (int x = 0; x < 2; ++x) {  // 32-byte stores: whole sectors of this row
+                        uint32_t v[8];
+#pragma unroll
+                        for (int y = 0; y < 8; ++y)
+                            v[y] = pack_bf16x2(__uint_as_float(o[16 * x + 2 * y]) * inv,
+                                               __uint_as_float(o[16 * x + 2 * y + 1]) * inv);
+                        st_global_v8(orow + c * 4 + 2 * x, v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7]);
                     }
                 }
                 if (half == 0) p.lse[tok * kRows + r] = (m_run + log2f(l)) * kLn2;

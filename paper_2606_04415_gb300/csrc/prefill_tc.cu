@@ -499,14 +499,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
                     tc::tmem_wait_ld();
                     if (row_ok) {
+                        // 32-byte stores: whole sectors of this row
 #pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            uint4 v;
-                            v.x = pack_bf16x2(__uint_as_float(o[8 * j + 0]) * inv, __uint_as_float(o[8 * j + 1]) * inv);
-                            v.y = pack_bf16x2(__uint_as_float(o[8 * j + 2]) * inv, __uint_as_float(o[8 * j + 3]) * inv);
-                            v.z = pack_bf16x2(__uint_as_float(o[8 * j + 4]) * inv, __uint_as_float(o[8 * j + 5]) * inv);
-                            v.w = pack_bf16x2(__uint_as_float(o[8 * j + 6]) * inv, __uint_as_float(o[8 * j + 7]) * inv);
-                            orow[c * 4 + j] = v;
+                        for (int j = 0; j < 2; ++j) {
+                            uint32_t v[8];
+#pragma unroll
+                            for (int x = 0; x < 8; ++x)
+                                v[x] = pack_bf16x2(__uint_as_float(o[16 * j + 2 * x]) * inv,
+                                                   __uint_as_float(o[16 * j + 2 * x + 1]) * inv);
+                            st_global_v8(orow + c * 4 + 2 * j, v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7]);
                         }
                     }
                 }
