@@ -22,20 +22,28 @@ __global__ void __launch_bounds__(256) kv_append_kernel(
     const int64_t total = static_cast<int64_t>(num_tokens) * per_tok;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t t = i / per_tok;
-        const int32_t c = static_cast<int32_t>(i - t * per_tok);
+        int64_t t;
+        int32_t c;
+        if (total < (1LL << 31)) {  // 32-bit division at step sizes
+            const uint32_t t32 = static_cast<uint32_t>(i) / static_cast<uint32_t>(per_tok);
+            t = t32;
+            c = static_cast<int32_t>(static_cast<uint32_t>(i) - t32 * static_cast<uint32_t>(per_tok));
+        } else {
+            t = i / per_tok;
+            c = static_cast<int32_t>(i - t * per_tok);
+        }
+        // the new row and its slot are independent loads: both in flight at once
+        const bool is_k = c < k_chunks;
+        const int32_t cv = c - k_chunks;
+        const uint4 v = is_k ? __ldg(k_new + t * k_chunks + c) : __ldg(v_new + t * v_chunks + cv);
         const int64_t s = __ldg(slots + t);
         if (s < 0) continue;
         if (s >= num_slots) {
             if (c == 0) atomicOr(&g_device_error, 1);
             continue;
         }
-        if (c < k_chunks) {
-            k_cache[s * k_chunks + c] = __ldg(k_new + t * k_chunks + c);
-        } else {
-            const int32_t cv = c - k_chunks;
-            v_cache[s * v_chunks + cv] = __ldg(v_new + t * v_chunks + cv);
-        }
+        if (is_k) k_cache[s * k_chunks + c] = v;
+        else v_cache[s * v_chunks + cv] = v;
     }
 }
 

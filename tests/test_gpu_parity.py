@@ -387,3 +387,30 @@ def test_decode_long_token_many_splits():
     assert st.plan.info()["decode_items"] >= 64
     out, lse = st.results()
     _compare(batch, out, lse)
+
+
+def test_decode_longest_context_split_cap():
+    """A 100000-key decode beside short ones: items of 448 keys (the planner
+    keeps a token to at most 256 splits), about 224 partials merged in seven
+    32-split chunks."""
+    sh = W.SHAPES["qwen"]
+    ql, ctx, ph = [1, 1, 1], [100000, 1000, 17], [1, 1, 1]
+    rng = np.random.default_rng(930)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="longest_decode")
+    st = _step(batch)
+    assert st.plan.info()["decode_items"] > 200
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_mla_longest_context():
+    """A 131072-key latent decode and a short prefill: about 128 pieces of
+    16 tiles, merged in four 32-split chunks at d_v 512."""
+    sh = W.Shape(128, 1, 576, 512, 64, True)
+    ql, ctx, ph = [1, 9], [131072, 9], [1, 0]
+    rng = np.random.default_rng(940)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_longest")
+    st = _step(batch)
+    assert st.plan.info()["prefill_items"] > 2 * 96
+    out, lse = st.results()
+    _compare(batch, out, lse)
