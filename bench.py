@@ -47,7 +47,7 @@ L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 # summaries with the commands are under profiles/. Set to None for a
 # workload whose kernels change until they are captured again.
 NCU_TRAFFIC = {
-    "qwen_coloc": 489.9e6,   # prefill_tc 33.4 MB + decode_tma 438.4 MB read + 18.1 MB write
+    "qwen_coloc": 490.0e6,   # prefill_tc 33.5 MB + decode_tma 438.4 MB read + 18.1 MB write
     "qwen_decode": 319.2e6,  # decode_tma 308.6 MB read + 10.6 MB write
 }
 
