@@ -259,8 +259,26 @@ def run_fnpu(args):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     flush_r = torch.zeros(L2_FLUSH_BYTES // 8, dtype=torch.float32, device=dev)
 
-    for _ in range(args.warmup):
+    # warm-up; with --dispatch feedback each warm-up step also feeds its phase
+    # times to the decode-share controller and the next step is planned with
+    # the share it returns (Sec. 3.4 dispatch ratio)
+    share = args.decode_share if args.decode_share > 0 else 24
+    trace = []
+    for w in range(args.warmup):
+        if args.dispatch == "feedback":
+            _flush_l2(flush, flush_r)
         st.run()
+        if args.dispatch == "feedback" and w > 0:  # the first run is cold (module load, first touch)
+            try:
+                pre_ms, dec_ms = fnpu.plan_phase_ms(st.plan)
+            except fnpu.FnpuError:  # one phase only: nothing to balance
+                break
+            nxt = fnpu.dispatch_next_share(share, pre_ms, dec_ms)
+            trace.append([share, round(pre_ms * 1e3, 1), round(dec_ms * 1e3, 1)])
+            if nxt != share:
+                share = nxt
+                st.replan(fnpu.PlanOpts(args.split, share, 0, args.flags))
+                info = st.plan.info()
     torch.cuda.synchronize(dev)
     if fnpu.plan_check(st.plan) != fnpu.FNPU_OK or fnpu.check() != fnpu.FNPU_OK:
         raise RuntimeError("device error flag raised during warm-up")
@@ -344,7 +362,7 @@ def run_fnpu(args):
         "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T,
                    "num_seqs": batch.num_seqs, "prefill_ctx": int(batch.context_len[0]),
                    "flops": F, "bytes": work["bytes"], "l2": "flushed between timed steps (512 MB write, then 256 MB read)",
-                   "plan": info},
+                   "plan": info, "dispatch": args.dispatch},
         "roofline": roof,
         "roofline_step_frac": {"burst": step_roof / (step_ms * 1e-3),
                                "sustained": step_roof_sus / (step_ms * 1e-3),
@@ -355,6 +373,9 @@ def run_fnpu(args):
         "gpu_launches": K * (1 + info["launches_per_run"]),
         "clocks": clk,
     }
+    if args.dispatch == "feedback":
+        line["config"]["decode_share_pct"] = share
+        line["config"]["dispatch_trace"] = trace  # [share %, prefill us, decode us] per warm-up step
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(batch, target_seconds=args.ref_seconds)
     elif rank == 0:
@@ -377,6 +398,9 @@ def main(argv=None):
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--split", type=int, default=0, help="decode split keys (0 = planner)")
     ap.add_argument("--decode-share", type=int, default=0)
+    ap.add_argument("--dispatch", default="feedback", choices=["planner", "feedback"],
+                    help="decode share of a co-located step: the phase-time feedback loop run over "
+                         "the warm-up steps (default), or the planner's model alone")
     ap.add_argument("--flags", type=int, default=0)
     ap.add_argument("--ref-seconds", type=float, default=15.0)
     ap.add_argument("--traffic", type=float, default=None,

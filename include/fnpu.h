@@ -163,6 +163,36 @@ int fnpu_plan_info(const fnpu_plan *plan, int32_t *prefill_items, int32_t *decod
                    int32_t *launches_per_run, int64_t *workspace_bytes);
 
 /*
+ * Dispatch-ratio feedback (Sec. 3.4: the phase-aware dispatcher sets the
+ * share of the device that serves decode from the measured pressure of each
+ * phase). A serving loop plans step n with fnpu_plan_opts.decode_share_pct =
+ * s_n, runs it, reads the phase times, and plans step n + 1 with the share
+ * the controller returns.
+ *
+ * fnpu_plan_phase_ms: for a co-located plan (both phases present, launched
+ * side by side), the device time from the start of the last run of `plan` to
+ * the end of its prefill work (*prefill_ms) and to the end of its decode work
+ * including the split merge (*decode_ms). Blocks until that run has ended.
+ *   Errors: FNPU_EINVAL for NULL arguments or a plan that has not run yet;
+ *   FNPU_EUNSUPPORTED for a plan that does not co-locate (one phase only,
+ *   latent attention, or FNPU_PLAN_SEPARATE_LAUNCHES).
+ *
+ * fnpu_dispatch_next_share: host arithmetic only. From the share share_pct
+ * (1..99, percent of SMs, as decode_share_pct) and the phase times it gave,
+ * the share for the next step: with decode time taken as proportional to
+ * 1 / share and prefill time to 1 / (100 - share), the share at which both
+ * phases would end together, approached halfway (at least one point while
+ * that share is a point or more away) and clamped to [1, 50]; kept when
+ * |decode - prefill| <= tolerance * the larger, or when the share is within
+ * a point of the balance share.
+ *   Errors: FNPU_EINVAL for a NULL out pointer, a share outside 1..99, a
+ *   time that is not positive, or a negative tolerance.
+ */
+int fnpu_plan_phase_ms(const fnpu_plan *plan, float *prefill_ms, float *decode_ms);
+int fnpu_dispatch_next_share(int32_t share_pct, float prefill_ms, float decode_ms, float tolerance,
+                             int32_t *next_share_pct);
+
+/*
  * Decode attention without any allocation. The paper has no counterpart:
  * this entry point exists for callers that may not call cudaMalloc at all,
  * for instance code that must stay inside memory another framework reserved

@@ -38,7 +38,8 @@ PLAN_NO_TCGEN05 = 2
 EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
-    "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error",
+    "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error", "fnpu_plan_phase_ms",
+    "fnpu_dispatch_next_share",
 )
 
 
@@ -99,9 +100,13 @@ def load(build_if_missing: bool = True):
     lib.fnpu_last_cuda_error.restype = ctypes.c_char_p
     lib.fnpu_status_str.argtypes = [ctypes.c_int]
     lib.fnpu_status_str.restype = ctypes.c_char_p
+    lib.fnpu_plan_phase_ms.argtypes = [P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_float)]
+    lib.fnpu_dispatch_next_share.argtypes = [i32, ctypes.c_float, ctypes.c_float, ctypes.c_float,
+                                             ctypes.POINTER(i32)]
     for name in ("fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex",
                  "fnpu_mixed_attn_run", "fnpu_plan_check", "fnpu_check", "fnpu_plan_info",
-                 "fnpu_version", "fnpu_decode_attn_noalloc"):
+                 "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_plan_phase_ms",
+                 "fnpu_dispatch_next_share"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -241,3 +246,22 @@ def check(stream=None) -> int:
 
 def version() -> int:
     return int(load().fnpu_version())
+
+
+def plan_phase_ms(plan: Plan) -> tuple:
+    """(prefill_ms, decode_ms) of the last co-located run of `plan`."""
+    a, b = ctypes.c_float(), ctypes.c_float()
+    rc = load().fnpu_plan_phase_ms(plan.handle, ctypes.byref(a), ctypes.byref(b))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_plan_phase_ms")
+    return a.value, b.value
+
+
+def dispatch_next_share(share_pct: int, prefill_ms: float, decode_ms: float, tolerance: float = 0.05) -> int:
+    """Decode share (percent of SMs) for the next step of a serving loop."""
+    out = ctypes.c_int32()
+    rc = load().fnpu_dispatch_next_share(int(share_pct), float(prefill_ms), float(decode_ms), float(tolerance),
+                                         ctypes.byref(out))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_dispatch_next_share")
+    return out.value

@@ -12,6 +12,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <mutex>
 #include <set>
 #include <utility>
@@ -552,10 +553,10 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         if (cudaDeviceGetStreamPriorityRange(&lo, &hi) != cudaSuccess ||
             cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess ||
             cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess ||
-            cudaEventCreateWithFlags(&pl->e_fork, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pl->e_fork, cudaEventDefault) != cudaSuccess ||
             cudaEventCreateWithFlags(&pl->e_started, cudaEventDisableTiming) != cudaSuccess ||
-            cudaEventCreateWithFlags(&pl->e_pre, cudaEventDisableTiming) != cudaSuccess ||
-            cudaEventCreateWithFlags(&pl->e_dec, cudaEventDisableTiming) != cudaSuccess) {
+            cudaEventCreateWithFlags(&pl->e_pre, cudaEventDefault) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pl->e_dec, cudaEventDefault) != cudaSuccess) {
             cudaGetLastError();
             destroy_sync_objects(pl);
             delete pl;
@@ -755,6 +756,51 @@ int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_
     if (launches_per_run)
         *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0) + (pl->num_mgroups > 0);
     if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_bytes);
+    return FNPU_OK;
+}
+
+// Phase times of the last co-located run: the fork, prefill-end and
+// decode-end events of the plan's two streams carry device timestamps.
+int fnpu_plan_phase_ms(const fnpu_plan *pl, float *prefill_ms, float *decode_ms) {
+    if (!pl || !prefill_ms || !decode_ms) return FNPU_EINVAL;
+    if (!pl->coloc) return FNPU_EUNSUPPORTED;
+    if (cudaEventSynchronize(pl->e_pre) != cudaSuccess || cudaEventSynchronize(pl->e_dec) != cudaSuccess)
+        return cuda_fail(cudaGetLastError(), "cudaEventSynchronize (phase times)");
+    float a = 0.f, b = 0.f;
+    if (cudaEventElapsedTime(&a, pl->e_fork, pl->e_pre) != cudaSuccess ||
+        cudaEventElapsedTime(&b, pl->e_fork, pl->e_dec) != cudaSuccess) {
+        cudaGetLastError();  // no run of this plan has been recorded yet
+        return FNPU_EINVAL;
+    }
+    *prefill_ms = a;
+    *decode_ms = b;
+    return FNPU_OK;
+}
+
+// Dispatch-ratio feedback (Sec. 3.4): while each phase holds its own SMs,
+// decode time goes about as 1 / s and prefill time as 1 / (1 - s) for a
+// decode share s of the SMs, so times d and p measured at share s give
+// D = d s and P = p (1 - s), and both phases would end together at
+// s* = D / (D + P). The next share moves halfway there (a damped step, as the
+// prefill time is a step function of its SM count), at least one point while
+// s* is a point or more away, and stays within [1, 50] percent.
+int fnpu_dispatch_next_share(int32_t share_pct, float prefill_ms, float decode_ms, float tolerance,
+                             int32_t *next_share_pct) {
+    if (!next_share_pct || share_pct < 1 || share_pct > 99 || !(prefill_ms > 0.f) || !(decode_ms > 0.f) ||
+        !(tolerance >= 0.f))
+        return FNPU_EINVAL;
+    auto clamp = [](int32_t v) { return std::min<int32_t>(50, std::max<int32_t>(1, v)); };
+    const double p = prefill_ms, d = decode_ms;
+    if (std::fabs(d - p) <= tolerance * std::max(d, p)) {
+        *next_share_pct = clamp(share_pct);
+        return FNPU_OK;
+    }
+    const double s = share_pct / 100.0;
+    const double dd = d * s, pp = p * (1.0 - s);
+    const double target = dd / (dd + pp);
+    int32_t next = static_cast<int32_t>(std::lround(100.0 * (s + 0.5 * (target - s))));
+    if (next == share_pct && std::fabs(100.0 * target - share_pct) >= 1.0) next += d > p ? 1 : -1;
+    *next_share_pct = clamp(next);
     return FNPU_OK;
 }
 

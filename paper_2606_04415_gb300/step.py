@@ -46,6 +46,13 @@ class DeviceStep:
         self.plan = mixed_attn_plan(self.desc, batch.query_len, batch.context_len, batch.phase,
                                     batch.block_table, opts=opts)
 
+    def replan(self, opts: Optional[PlanOpts] = None):
+        """Plan the same batch again with other options (for instance the
+        decode share a dispatch controller chose for the next step)."""
+        self.plan.destroy()
+        b = self.batch
+        self.plan = mixed_attn_plan(self.desc, b.query_len, b.context_len, b.phase, b.block_table, opts=opts)
+
     def append(self, stream=None):
         kv_append(self.desc, self.k_new, self.v_new, self.slot_mapping, self.k_cache, self.v_cache,
                   stream=stream)

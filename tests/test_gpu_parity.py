@@ -414,3 +414,47 @@ def test_mla_longest_context():
     assert st.plan.info()["prefill_items"] > 2 * 96
     out, lse = st.results()
     _compare(batch, out, lse)
+
+
+def test_dispatch_feedback_loop_on_colocated_steps():
+    """Phase times of co-located runs feed the decode-share controller for a
+    few steps (the dispatch ratio of Sec. 3.4); each step's plan uses the
+    share the last one chose, and the output stays correct."""
+    import paper_2606_04415_gb300 as fnpu
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(950)
+    ql = [512] + [1] * 48
+    ctx = [512 + 3000] + rng.integers(200, 6000, size=48).tolist()
+    ph = [0] + [1] * 48
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="dispatch_loop")
+    share = 24
+    st = _step(batch, share=share)
+    shares = [share]
+    for _ in range(4):
+        pre, dec = fnpu.plan_phase_ms(st.plan)
+        assert 0 < pre < 1000 and 0 < dec < 1000
+        share = fnpu.dispatch_next_share(share, pre, dec)
+        assert 1 <= share <= 50
+        shares.append(share)
+        st.replan(fnpu.PlanOpts(0, share, 0, 0))
+        st.attend()
+        assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
+    out, lse = st.results()
+    _compare(batch, out, lse)
+
+
+def test_phase_times_need_a_colocated_plan_that_ran():
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(960)
+    dec_only = W.build_batch(sh, [1, 1], [700, 90], [1, 1], rng, name="dec_only")
+    st = _step(dec_only)
+    with pytest.raises(fnpu.FnpuError) as e:
+        fnpu.plan_phase_ms(st.plan)
+    assert e.value.code == fnpu.FNPU_EUNSUPPORTED
+    mixed = W.build_batch(sh, [300, 1], [300, 900], [0, 1], rng, name="mixed_unrun")
+    fresh = DeviceStep(mixed)  # planned, never run
+    with pytest.raises(fnpu.FnpuError) as e:
+        fnpu.plan_phase_ms(fresh.plan)
+    assert e.value.code == fnpu.FNPU_EINVAL
