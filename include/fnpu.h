@@ -106,12 +106,14 @@ int fnpu_kv_append(const fnpu_attn_desc *desc, const void *k_new, const void *v_
 /*
  * Build the work list for one step. Host arrays, all of length num_seqs:
  *   query_len[s] >= 1, context_len[s] >= query_len[s],
- *   phase[s] = 0 (prefill chunk) or 1 (decode; requires query_len[s] == 1),
+ *   phase[s] = 0 (prefill chunk) or 1 (decode),
  *   block_table: int32 [num_seqs, block_table_stride]; only the first
  *   ceil(context_len[s] / bs) entries of row s are read, each < num_blocks.
  * The phase decides only which queue a sequence's work enters (prefill tiles
  * on the tensor-core path, decode split items on the bandwidth path), never
- * the result. The plan copies everything it needs (the block table included)
+ * the result. A decode of several tokens (query_len[s] > 1, as in speculative
+ * verification) is causal attention of a short chunk on its context and
+ * takes the prefill path; one-token decodes take the decode path. The plan copies everything it needs (the block table included)
  * to its own device workspace with one asynchronous copy on `stream`; the
  * host arrays may be freed on return. The plan stays valid for any number of
  * runs with the same metadata and caches of the same shape.

@@ -299,9 +299,10 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         const int32_t q = query_len[s], c = context_len[s];
         if (q < 1 || c < q) return FNPU_EINVAL;
         if (phase[s] > 1) return FNPU_EINVAL;
-        if (phase[s] == 1 && q != 1) return FNPU_EINVAL;
-        has_decode |= phase[s] == 1;
-        has_prefill |= phase[s] == 0;
+        // a decode step of several tokens (speculative verification) is causal
+        // attention of a short chunk: its rows take the prefill path
+        has_decode |= phase[s] == 1 && q == 1;
+        has_prefill |= phase[s] == 0 || q > 1;
         const int32_t nb = (c + bs - 1) / bs;
         if (nb > block_table_stride) return FNPU_EINVAL;
         for (int32_t j = 0; j < nb; ++j) {
@@ -356,9 +357,11 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     // bytes; about four items per CTA keep that close to the mean (a TMA
     // decode item streams every kv head of its keys). The per-head kernel
     // aims at about 3 waves of 2 CTAs per SM.
+    // the queue a sequence's work enters: decode items for one-token decodes
+    auto decode_queue = [&](int32_t s) { return phase[s] == 1 && query_len[s] == 1; };
     int64_t dec_keys = 0;
     for (int32_t s = 0; s < num_seqs; ++s)
-        if (phase[s] == 1)
+        if (decode_queue(s))
             dec_keys += static_cast<int64_t>(context_len[s]) * (pl->use_dt ? 1 : desc->num_kv_heads);
     int32_t split = o.decode_split_keys;
     if (split == 0) {
@@ -436,7 +439,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                                                  0, 0, 0});
                 }
             }
-        } else if (phase[s] == 1 && pl->use_dt) {
+        } else if (decode_queue(s) && pl->use_dt) {
             // items over all kv heads; a split sequence is merged by the merge
             // kernel (at most 256 splits: its scratch grows with them)
             const int32_t sk = std::max(split, (c + 256 * 64 - 1) / (256 * 64) * 64);
@@ -450,7 +453,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 const int32_t kb = sp * sk, ke = std::min(c, kb + sk);
                 ditems.push_back(DecodeItem{s, 0, kb, ke, sp, ns, base, 0});
             }
-        } else if (phase[s] == 1) {
+        } else if (decode_queue(s)) {
             const int32_t ns = (c + split - 1) / split;
             for (int32_t kvh = 0; kvh < desc->num_kv_heads; ++kvh) {
                 const int32_t grp = groups++;

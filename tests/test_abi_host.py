@@ -57,7 +57,7 @@ QWEN = dict(num_q_heads=28, num_kv_heads=4, head_dim_qk=128, head_dim_v=128, blo
 
 
 @pytest.mark.parametrize("case", [
-    "ctx_lt_q", "q_zero", "decode_q2", "phase_2", "block_oob", "block_neg", "stride_short",
+    "ctx_lt_q", "q_zero", "phase_2", "block_oob", "block_neg", "stride_short",
 ])
 def test_plan_rejects_bad_metadata(case):
     desc = fnpu.make_desc(**QWEN)
@@ -67,8 +67,6 @@ def test_plan_rejects_bad_metadata(case):
         cl = [3, 40]
     elif case == "q_zero":
         ql = [0, 1]
-    elif case == "decode_q2":
-        ql = [4, 2]
     elif case == "phase_2":
         ph = [0, 2]
     elif case == "block_oob":
@@ -78,6 +76,15 @@ def test_plan_rejects_bad_metadata(case):
     elif case == "stride_short":
         bt = np.zeros((2, 2), np.int32)
     assert _plan_rc(desc, ql, cl, ph, bt) == fnpu.FNPU_EINVAL
+
+
+def test_plan_accepts_multi_token_decode():
+    """A decode of several tokens (speculative verification) is valid
+    metadata: without a GPU the plan then fails on the device, not on the
+    arguments."""
+    desc = fnpu.make_desc(**QWEN)
+    bt = np.zeros((2, 4), np.int32)
+    assert _plan_rc(desc, [4, 3], [10, 40], [0, 1], bt) != fnpu.FNPU_EINVAL
 
 
 def test_plan_rejects_bad_shape_and_options():

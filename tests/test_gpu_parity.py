@@ -458,3 +458,30 @@ def test_phase_times_need_a_colocated_plan_that_ran():
     with pytest.raises(fnpu.FnpuError) as e:
         fnpu.plan_phase_ms(fresh.plan)
     assert e.value.code == fnpu.FNPU_EINVAL
+
+
+@pytest.mark.parametrize("flags", [0, NO_TC])
+def test_multi_token_decode(flags):
+    """Decode steps of several tokens (speculative verification of 2, 4 and 7
+    draft tokens) beside one-token decodes and a prefill chunk: the
+    multi-token rows take the prefill path with their causal mask; every row
+    against the oracle."""
+    sh = W.SHAPES["qwen"]
+    ql = [2, 4, 7, 1, 1, 300]
+    ctx = [2000, 513, 4096 + 7, 1000, 77, 300 + 900]
+    ph = [1, 1, 1, 1, 1, 0]
+    rng = np.random.default_rng(970)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="multi_token_decode")
+    out, lse = _step(batch, flags=flags).results()
+    _compare(batch, out, lse)
+
+
+def test_mla_multi_token_decode():
+    """A three-token latent decode (speculative verification) beside a
+    one-token one."""
+    sh = W.Shape(128, 1, 576, 512, 64, True)
+    ql, ctx, ph = [3, 1], [1500, 700], [1, 1]
+    rng = np.random.default_rng(980)
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_multi_token")
+    out, lse = _step(batch).results()
+    _compare(batch, out, lse)
