@@ -82,6 +82,10 @@ typedef struct {
 
 #define FNPU_PLAN_SEPARATE_LAUNCHES 1 /* run prefill and decode as separate launches */
 #define FNPU_PLAN_NO_TCGEN05 2        /* prefill on the mma.sync path (comparison only) */
+#define FNPU_PLAN_GREEN_CONTEXTS 4    /* co-located step: prefill and decode in green contexts
+                                         over disjoint SM partitions (the decode share rounded
+                                         up to the device's partition granularity); plan
+                                         fails with FNPU_EUNSUPPORTED where they cannot be made */
 
 /*
  * KV append: for each token t in [0, num_tokens) with slot_mapping[t] >= 0,

@@ -34,6 +34,7 @@ FNPU_EDEVICE_RANGE = -6
 
 PLAN_SEPARATE_LAUNCHES = 1
 PLAN_NO_TCGEN05 = 2
+PLAN_GREEN_CONTEXTS = 4
 
 EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",

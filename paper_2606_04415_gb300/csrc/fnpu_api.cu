@@ -15,8 +15,11 @@
 #include <cmath>
 #include <mutex>
 #include <set>
+#include <type_traits>
 #include <utility>
 #include <vector>
+
+#include <cuda.h>
 
 #include "fnpu_internal.h"
 
@@ -59,6 +62,10 @@ struct fnpu_plan {
     int32_t pre_ctas = 0;
     cudaStream_t s_pre = nullptr, s_dec = nullptr;
     cudaEvent_t e_fork = nullptr, e_started = nullptr, e_pre = nullptr, e_dec = nullptr;
+    // FNPU_PLAN_GREEN_CONTEXTS: the two streams belong to green contexts over
+    // disjoint SM partitions (dec_sms SMs for decode, pre_ctas for prefill)
+    CUgreenCtx g_pre = nullptr, g_dec = nullptr;
+    int32_t dec_sms = 0;
 };
 
 namespace fnpu {
@@ -75,9 +82,46 @@ namespace {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Driver entry points of green contexts (SM partitions), looked up once.
+struct GreenApi {
+    CUresult (*device_get)(CUdevice *, int) = nullptr;
+    CUresult (*get_resource)(CUdevice, CUdevResource *, CUdevResourceType) = nullptr;
+    CUresult (*split)(CUdevResource *, unsigned int *, const CUdevResource *, CUdevResource *, unsigned int,
+                      unsigned int) = nullptr;
+    CUresult (*gen_desc)(CUdevResourceDesc *, CUdevResource *, unsigned int) = nullptr;
+    CUresult (*create)(CUgreenCtx *, CUdevResourceDesc, CUdevice, unsigned int) = nullptr;
+    CUresult (*destroy)(CUgreenCtx) = nullptr;
+    CUresult (*stream_create)(CUstream *, CUgreenCtx, unsigned int, int) = nullptr;
+    bool ok = false;
+};
+
+const GreenApi &green_api() {
+    static std::once_flag once;
+    static GreenApi g;
+    std::call_once(once, [] {
+        auto get = [](const char *name, auto &fn) {
+            void *ptr = nullptr;
+            cudaDriverEntryPointQueryResult q;
+            if (cudaGetDriverEntryPointByVersion(name, &ptr, 13000, cudaEnableDefault, &q) == cudaSuccess &&
+                q == cudaDriverEntryPointSuccess)
+                fn = reinterpret_cast<std::remove_reference_t<decltype(fn)>>(ptr);
+            return fn != nullptr;
+        };
+        g.ok = get("cuDeviceGet", g.device_get) && get("cuDeviceGetDevResource", g.get_resource) &&
+               get("cuDevSmResourceSplitByCount", g.split) && get("cuDevResourceGenerateDesc", g.gen_desc) &&
+               get("cuGreenCtxCreate", g.create) && get("cuGreenCtxDestroy", g.destroy) &&
+               get("cuGreenCtxStreamCreate", g.stream_create);
+        cudaGetLastError();
+    });
+    return g;
+}
+
 void destroy_sync_objects(fnpu_plan *pl) {
     if (pl->s_pre) cudaStreamDestroy(pl->s_pre);
     if (pl->s_dec) cudaStreamDestroy(pl->s_dec);
+    if (pl->g_pre) green_api().destroy(pl->g_pre);
+    if (pl->g_dec) green_api().destroy(pl->g_dec);
+    pl->g_pre = pl->g_dec = nullptr;
     if (pl->e_started) cudaEventDestroy(pl->e_started);
     if (pl->e_dec) cudaEventDestroy(pl->e_dec);
     if (pl->e_fork) cudaEventDestroy(pl->e_fork);
@@ -506,6 +550,38 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                               ? std::min(sms - 1, std::max(1, (sms * o.decode_share_pct + 50) / 100))
                               : choose_decode_sms(item_tiles, tile_scale, dec_bytes, sms);
         pl->pre_ctas = sms - k;
+        if (o.flags & FNPU_PLAN_GREEN_CONTEXTS) {
+            // enforce the split in hardware: a green context of at least k SMs
+            // (rounded up to the partition granularity) for decode and one of
+            // the remaining SMs for prefill, each with its own stream
+            const GreenApi &g = green_api();
+            int dev = 0;
+            CUdevice cudev = 0;
+            CUdevResource all{}, part{}, rest{};
+            CUdevResourceDesc d_dec = nullptr, d_pre = nullptr;
+            unsigned int ngroups = 1;
+            CUstream st_dec = nullptr, st_pre = nullptr;
+            const bool made = g.ok && cudaGetDevice(&dev) == cudaSuccess && g.device_get(&cudev, dev) == CUDA_SUCCESS &&
+                              g.get_resource(cudev, &all, CU_DEV_RESOURCE_TYPE_SM) == CUDA_SUCCESS &&
+                              static_cast<int32_t>(all.sm.smCount) == sms &&
+                              g.split(&part, &ngroups, &all, &rest, 0, static_cast<unsigned int>(k)) == CUDA_SUCCESS &&
+                              ngroups == 1 && rest.sm.smCount > 0 && g.gen_desc(&d_dec, &part, 1) == CUDA_SUCCESS &&
+                              g.gen_desc(&d_pre, &rest, 1) == CUDA_SUCCESS &&
+                              g.create(&pl->g_dec, d_dec, cudev, CU_GREEN_CTX_DEFAULT_STREAM) == CUDA_SUCCESS &&
+                              g.create(&pl->g_pre, d_pre, cudev, CU_GREEN_CTX_DEFAULT_STREAM) == CUDA_SUCCESS &&
+                              g.stream_create(&st_dec, pl->g_dec, CU_STREAM_NON_BLOCKING, 0) == CUDA_SUCCESS &&
+                              g.stream_create(&st_pre, pl->g_pre, CU_STREAM_NON_BLOCKING, 0) == CUDA_SUCCESS;
+            pl->s_dec = reinterpret_cast<cudaStream_t>(st_dec);
+            pl->s_pre = reinterpret_cast<cudaStream_t>(st_pre);
+            if (!made) {
+                cudaGetLastError();
+                destroy_sync_objects(pl);
+                delete pl;
+                return FNPU_EUNSUPPORTED;
+            }
+            pl->dec_sms = static_cast<int32_t>(part.sm.smCount);
+            pl->pre_ctas = static_cast<int32_t>(rest.sm.smCount);
+        }
     }
     int32_t pparts = 0, pgroups = 0;
     if (!tc_units.empty()) {
@@ -553,9 +629,10 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->num_pgroups = pgroups;
     if (pl->coloc) {
         int lo = 0, hi = 0;
+        const bool green = pl->g_pre != nullptr;  // streams already made in the partitions
         if (cudaDeviceGetStreamPriorityRange(&lo, &hi) != cudaSuccess ||
-            cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess ||
-            cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess ||
+            (!green && cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess) ||
+            (!green && cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess) ||
             cudaEventCreateWithFlags(&pl->e_fork, cudaEventDefault) != cudaSuccess ||
             cudaEventCreateWithFlags(&pl->e_started, cudaEventDisableTiming) != cudaSuccess ||
             cudaEventCreateWithFlags(&pl->e_pre, cudaEventDefault) != cudaSuccess ||
@@ -704,10 +781,11 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
         cudaStream_t s = static_cast<cudaStream_t>(stream);
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
         FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
-        int rc = launch_prefill_tc(p, pl->s_pre, pl->pre_ctas, pl->e_started);
+        const bool green = pl->g_pre != nullptr;  // partitions enforced: no placement order to keep
+        int rc = launch_prefill_tc(p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
         if (rc == FNPU_OK) {
-            FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_started, 0));
-            rc = launch_decode_tma(p, pl->s_dec, 3 * pl->num_sms);
+            FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, green ? pl->e_fork : pl->e_started, 0));
+            rc = launch_decode_tma(p, pl->s_dec, 3 * (green ? pl->dec_sms : pl->num_sms));
         }
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));

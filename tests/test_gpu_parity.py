@@ -485,3 +485,27 @@ def test_mla_multi_token_decode():
     batch = W.build_batch(sh, ql, ctx, ph, rng, name="mla_multi_token")
     out, lse = _step(batch).results()
     _compare(batch, out, lse)
+
+
+GREEN = 4  # FNPU_PLAN_GREEN_CONTEXTS
+
+
+@pytest.mark.parametrize("share", [0, 20])
+def test_green_context_partitions(share):
+    """Co-location with the SM split enforced by green contexts (disjoint SM
+    partitions for the two phases) gives the results of separate launches;
+    the dispatch feedback works on such plans too."""
+    import paper_2606_04415_gb300 as fnpu
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(77)
+    ql = [300, 1, 1, 129, 1] + [1] * 12
+    ctx = [300 + 2000, 700, 1500, 129 + 40, 33] + list(rng.integers(20, 3000, size=12))
+    ph = [0, 1, 1, 0, 1] + [1] * 12
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="coloc_green")
+    st = _step(batch, share=share, flags=GREEN)
+    a_out, a_lse = st.results()
+    b_out, b_lse = _step(batch, flags=SEPARATE).results()
+    _compare(batch, a_out, a_lse)
+    assert np.abs(a_out - b_out).max() <= O_TOL and np.abs(a_lse - b_lse).max() <= LSE_TOL
+    pre, dec = fnpu.plan_phase_ms(st.plan)
+    assert pre > 0 and dec > 0
