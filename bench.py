@@ -47,8 +47,8 @@ L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 # summaries with the commands are under profiles/. Set to None for a
 # workload whose kernels change until they are captured again.
 NCU_TRAFFIC = {
-    "qwen_coloc": 490.0e6,   # prefill_tc 33.5 MB + decode_tma 438.4 MB read + 18.1 MB write
-    "qwen_decode": 319.2e6,  # decode_tma 308.6 MB read + 10.6 MB write
+    "qwen_coloc": 472.3e6,   # prefill_tc 33.3 MB + decode_tma 437.7 MB read + 1.3 MB write
+    "qwen_decode": 309.0e6,  # decode_tma 308.1 MB read + 0.8 MB write
 }
 
 
