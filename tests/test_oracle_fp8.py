@@ -1,0 +1,141 @@
+"""Pins of the fp8 (e4m3) KV-cache reference against the format definition and
+the bf16 oracle. No GPU."""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import fp8
+
+
+def test_e4m3_values_of_known_codes():
+    assert fp8.e4m3_value(0x00) == 0.0
+    assert fp8.e4m3_value(0x01) == 2.0 ** -9          # smallest subnormal
+    assert fp8.e4m3_value(0x07) == 7 * 2.0 ** -9       # largest subnormal
+    assert fp8.e4m3_value(0x08) == 2.0 ** -6           # smallest normal
+    assert fp8.e4m3_value(0x38) == 1.0
+    assert fp8.e4m3_value(0x44) == 3.0
+    assert fp8.e4m3_value(0x7E) == 448.0               # largest finite
+    assert np.isnan(fp8.e4m3_value(0x7F))
+    assert fp8.e4m3_value(0xB8) == -1.0
+    assert fp8.e4m3_value(0xFE) == -448.0
+
+
+def test_every_finite_value_rounds_to_its_own_code():
+    codes = np.arange(127, dtype=np.uint8)
+    vals = np.array([fp8.e4m3_value(int(c)) for c in codes], np.float32)
+    assert np.array_equal(fp8.e4m3_round(vals), codes)
+    assert np.array_equal(fp8.e4m3_round(-vals[1:]), codes[1:] | 0x80)
+
+
+def test_ties_go_to_the_even_code_and_large_values_saturate():
+    # 1.0625 lies halfway between 1.0 (code 56) and 1.125 (57); 1.1875 between 57 and 58
+    assert fp8.e4m3_round(np.float32(1.0625)) == 56
+    assert fp8.e4m3_round(np.float32(1.1875)) == 58
+    assert fp8.e4m3_round(np.float32(1.07)) == 57
+    # subnormal range: 2^-10 halfway between 0 and 2^-9, 3*2^-10 between codes 1 and 2
+    assert fp8.e4m3_round(np.float32(2.0 ** -10)) == 0
+    assert fp8.e4m3_round(np.float32(3 * 2.0 ** -10)) == 2
+    for big in (448.5, 463.9, 500.0, 1e30):
+        assert fp8.e4m3_round(np.float32(big)) == 0x7E
+        assert fp8.e4m3_round(np.float32(-big)) == 0xFE
+
+
+def _bf16(x):
+    return (np.asarray(x, np.float32).view(np.uint32) >> 16).astype(np.uint16)
+
+
+def test_row_quantisation_maps_amax_to_448_and_bounds_the_error():
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((64, 4, 128)).astype(np.float32) * 3
+    bits = _bf16(x)
+    xf = fp8.bf16_bits_to_f32(bits).astype(np.float64)
+    codes, scale = fp8.quantize_rows(bits)
+    amax = np.abs(xf).max(-1)
+    assert np.allclose(scale, amax / 448, rtol=1e-7)
+    argmax = np.abs(xf).argmax(-1)
+    top = np.take_along_axis(codes, argmax[..., None], -1)[..., 0]
+    assert np.all((top & 0x7F) == 0x7E)
+    deq = fp8.e4m3_decode(codes) * scale[..., None]
+    # half a step of the e4m3 grid: 2^-4 relative for normals, 2^-10 * scale absolute below
+    err = np.abs(deq - xf)
+    assert np.all(err <= np.maximum(np.abs(xf) * 2.0 ** -4, scale[..., None] * 2.0 ** -10) * 1.0001)
+    zero = fp8.quantize_rows(np.zeros((1, 128), np.uint16))
+    assert zero[1][0] == 1.0 and not zero[0].any()
+
+
+def test_layout_permutations_are_bijections_and_group_lane_operands():
+    assert sorted(fp8.kpos(np.arange(128)).tolist()) == list(range(128))
+    assert sorted(fp8.vpos(np.arange(16)).tolist()) == list(range(16))
+    for k in range(8):
+        for c in range(4):
+            cols = [16 * k + 2 * c, 16 * k + 2 * c + 1, 16 * k + 2 * c + 8, 16 * k + 2 * c + 9]
+            assert fp8.kpos(cols).tolist() == [32 * c + 4 * k + r for r in range(4)]
+    for c in range(4):
+        assert fp8.vpos([2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9]).tolist() == [4 * c + r for r in range(4)]
+
+
+def test_pack_unpack_round_trip_and_append():
+    rng = np.random.default_rng(4)
+    nb, hkv = 5, 4
+    kc = rng.integers(0, 256, (nb, 16, hkv, 128), dtype=np.uint8)
+    vc = rng.integers(0, 256, (nb, 16, hkv, 128), dtype=np.uint8)
+    ks = rng.random((nb, 16, hkv)).astype(np.float32)
+    vs = rng.random((nb, 16, hkv)).astype(np.float32)
+    kp, vp = fp8.pack_pools(kc, ks, vc, vs)
+    assert kp.size == nb * fp8.block_bytes(hkv)
+    back = fp8.unpack_pools(kp, vp, hkv)
+    for a, b in zip(back, (kc, ks, vc, vs)):
+        assert np.array_equal(a, b)
+    new_k = _bf16(rng.standard_normal((3, hkv, 128)))
+    new_v = _bf16(rng.standard_normal((3, hkv, 128)))
+    slots = np.array([17, -1, 79], np.int64)
+    kp2, vp2 = fp8.kv_append(kp, vp, new_k, new_v, slots, hkv)
+    k2, ks2, v2, vs2 = fp8.unpack_pools(kp2, vp2, hkv)
+    qk, sk = fp8.quantize_rows(new_k)
+    assert np.array_equal(k2[1, 1], qk[0]) and np.array_equal(ks2[4, 15], sk[2])
+    assert np.array_equal(k2[0], kc[0]) and np.array_equal(v2[2], vc[2])   # untouched blocks
+
+
+def test_decode_attention_closed_forms():
+    rng = np.random.default_rng(5)
+    hkv, hq = 4, 8
+    kc = rng.integers(0, 120, (2, 16, hkv, 128), dtype=np.uint8)
+    vc = rng.integers(0, 120, (2, 16, hkv, 128), dtype=np.uint8)
+    ks = np.full((2, 16, hkv), 0.5, np.float32)
+    vs = np.full((2, 16, hkv), 0.25, np.float32)
+    kp, vp = fp8.pack_pools(kc, ks, vc, vs)
+    q = _bf16(rng.standard_normal((1, hq, 128)))
+    out, lse = fp8.decode_attention([1], np.array([[1, 0]]), q, kp, vp, num_q_heads=hq, num_kv_heads=hkv)
+    k0 = fp8.e4m3_decode(kc[1, 0]) * 0.5
+    v0 = fp8.e4m3_decode(vc[1, 0]) * 0.25
+    qf = fp8.bf16_bits_to_f32(q)[0].astype(np.float64)
+    for h in range(hq):   # one key: the output is its value, the LSE its score
+        assert np.allclose(out[0, h], v0[h // 2])
+        assert np.isclose(lse[0, h], k0[h // 2] @ qf[h] / np.sqrt(128))
+
+
+def test_matches_the_bf16_oracle_when_every_scale_is_one():
+    """Rows whose amax is exactly 448 have scale 1, and e4m3 values are exact
+    in bf16: the fp8 reference must then equal the bf16 oracle on the
+    dequantised cache."""
+    rng = np.random.default_rng(6)
+    hkv, hq, nb = 4, 28, 6
+    vals = np.array([fp8.e4m3_value(c) for c in range(127)], np.float32)
+    def rows(n):
+        x = rng.choice(np.concatenate([vals, -vals[1:]]), size=(n, 16, hkv, 128)).astype(np.float32) / 64
+        x[..., 0] = 448.0
+        return x
+    kx, vx = rows(nb), rows(nb)
+    kc, ks = fp8.quantize_rows(_bf16(kx))
+    vc, vs = fp8.quantize_rows(_bf16(vx))
+    assert np.all(ks == 1.0) and np.all(vs == 1.0)
+    kp, vp = fp8.pack_pools(kc, ks, vc, vs)
+    ctx = np.array([37, 90, 5])
+    bt = np.array([[2, 4, 0, 0, 0, 0], [1, 3, 5, 0, 2, 4], [5, 0, 0, 0, 0, 0]], np.int32)
+    q = _bf16(rng.standard_normal((3, hq, 128)))
+    out, lse = fp8.decode_attention(ctx, bt, q, kp, vp, num_q_heads=hq, num_kv_heads=hkv)
+    kdq = _bf16(fp8.e4m3_decode(kc).astype(np.float32))
+    vdq = _bf16(fp8.e4m3_decode(vc).astype(np.float32))
+    ref_o, ref_l = oracle.attention(np.ones(3, np.int32), ctx, bt, q, kdq, vdq, num_q_heads=hq,
+                                    num_kv_heads=hkv, head_dim_qk=128, head_dim_v=128, block_size=16)
+    assert np.abs(out - ref_o).max() < 1e-12 and np.abs(lse - ref_l).max() < 1e-12
