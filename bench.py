@@ -13,6 +13,7 @@ region.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the fp64 oracle on the host cores
+  python bench.py --workload qwen_decode --kv-fp8   # decode over the FP8 (e4m3) cache
 
 Under torchrun each rank runs an independent replica (seed + rank): the path
 has no exchange step, so there is no collective on the data path.
@@ -211,14 +212,50 @@ def cpu_baseline(batch, target_seconds: float = 15.0, reps: int = 1):
             "sample_seconds": t_sample, "step_seconds_extrapolated": t_step}
 
 
+def cpu_baseline_fp8(batch, target_seconds: float = 15.0):
+    """Time the fp64 FP8 reference: the step's append (all new rows, on the
+    whole pool) and the decode attention of an evenly spaced sample of the
+    sequences, extrapolated to all of them by keys. The sampled sequences'
+    prefix rows are put into the reference pools first, untimed."""
+    from oracle import fp8 as F8
+    sh = batch.shape
+    init = W.stale_pool_bytes(batch.num_blocks * F8.block_bytes(sh.num_kv_heads), batch.seed)
+    ctx = batch.context_len.astype(np.int64)
+    # the reference decodes about 25k keys a second (d = 128, 28 heads) and
+    # fills its pools about 8 times slower: a tenth of the budget for the
+    # decode sample keeps the whole call near the budget; at least one sequence
+    want = max(1, min(batch.num_seqs, int(round(batch.num_seqs * min(1.0, 25000 * target_seconds / 10 / ctx.sum())))))
+    seqs = np.unique(np.linspace(0, batch.num_seqs - 1, want).round().astype(np.int64))
+    k, v, sl = W.prefix_rows(batch)
+    pre = ctx - batch.query_len
+    p0 = np.concatenate([[0], np.cumsum(pre)])
+    pi = np.concatenate([np.arange(p0[s], p0[s + 1]) for s in seqs])
+    kp, vp = F8.kv_append(init[0], init[1], k[pi], v[pi], sl[pi], sh.num_kv_heads)
+    t0 = time.perf_counter()
+    kp, vp = F8.kv_append(kp, vp, batch.k_new, batch.v_new, batch.slot_mapping, sh.num_kv_heads)
+    t_append = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    F8.decode_attention(ctx[seqs], batch.block_table[seqs], batch.q[batch.query_start[seqs]], kp, vp,
+                        num_q_heads=sh.num_q_heads, num_kv_heads=sh.num_kv_heads)
+    t_sample = time.perf_counter() - t0
+    frac = float(ctx[seqs].sum()) / float(ctx.sum())
+    t_step = t_append + t_sample / frac
+    return {"value": batch.num_tokens / t_step, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": (f"decode of {len(seqs)} of {batch.num_seqs} sequences ({frac:.3f} of the keys), "
+                       f"fp64 numpy FP8 reference; step time = full append + sample / key fraction"),
+            "sample_seconds": t_sample, "step_seconds_extrapolated": t_step}
+
+
 def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return 0
     batch = W.make_batch(args.workload, seed=args.seed)
+    if args.kv_fp8:
+        _fp8_workload_ok(batch)
     per = []
     for i in range(args.warmup + args.steps):
-        r = cpu_baseline(batch, target_seconds=args.ref_seconds)
+        r = (cpu_baseline_fp8 if args.kv_fp8 else cpu_baseline)(batch, target_seconds=args.ref_seconds)
         if i >= args.warmup:
             per.append(r)
     step_s = statistics.median(x["step_seconds_extrapolated"] for x in per)
@@ -226,13 +263,19 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": args.workload, "seed": args.seed},
+            "data": "synthetic", "config": {"workload": args.workload, "seed": args.seed,
+                                            "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": per[0]["cores"], "kind": "oracle",
                              "sample": per[0]["sample"]},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
     print(json.dumps(line), flush=True)
     return 0
+
+
+def _fp8_workload_ok(batch):
+    if not np.all((batch.query_len == 1) & (batch.phase == 1)):
+        raise SystemExit("--kv-fp8 needs a decode-only workload (qwen_decode)")
 
 
 def run_fnpu(args):
@@ -251,9 +294,14 @@ def run_fnpu(args):
     peaks = _peaks()
 
     batch = W.make_batch(args.workload, seed=args.seed + rank)
-    work = W.algorithmic_work(batch)
+    work = W.algorithmic_work(batch, kv_fp8=args.kv_fp8)
     opts = fnpu.PlanOpts(args.split, args.decode_share, 0, args.flags)
-    st = DeviceStep(batch, opts=opts, device=str(dev))
+    if args.kv_fp8:
+        _fp8_workload_ok(batch)
+        init = W.stale_pool_bytes(batch.num_blocks * fnpu.FP8_BLOCK_BYTES, batch.seed)
+        st = DeviceStep(batch, opts=opts, device=str(dev), kv_fp8=True, pool_init=init)
+    else:
+        st = DeviceStep(batch, opts=opts, device=str(dev))
     info = st.plan.info()
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
@@ -349,7 +397,8 @@ def run_fnpu(args):
     else:
         roof = {"bound": "hbm", "achieved": B_attn / t_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = args.traffic if args.traffic is not None else NCU_TRAFFIC.get(args.workload)
+    roof["traffic"] = args.traffic if args.traffic is not None else \
+        NCU_TRAFFIC.get(args.workload + ("_fp8" if args.kv_fp8 else ""))
     roof["peak_source"] = peaks["source"] + " burst"
     step_roof = max(F / (peaks["bf16_tflops"] * 1e12), work["bytes"] / (peaks["hbm_gbs"] * 1e9))
     step_roof_sus = max(F / (peaks["bf16_tflops_sustained"] * 1e12), work["bytes"] / (peaks["hbm_gbs"] * 1e9))
@@ -358,11 +407,12 @@ def run_fnpu(args):
     line = {
         "metric": METRIC, "value": job_throughput(ws, T, step_ms), "unit": UNIT, "n_gpus": ws,
         "steps": K, "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": "fp8-e4m3 KV, f16 products" if args.kv_fp8 else "bf16",
+        "data": "synthetic",
         "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T,
                    "num_seqs": batch.num_seqs, "prefill_ctx": int(batch.context_len[0]),
                    "flops": F, "bytes": work["bytes"], "l2": "flushed between timed steps (512 MB write, then 256 MB read)",
-                   "plan": info, "dispatch": args.dispatch},
+                   "plan": info, "dispatch": args.dispatch, "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16"},
         "roofline": roof,
         "roofline_step_frac": {"burst": step_roof / (step_ms * 1e-3),
                                "sustained": step_roof_sus / (step_ms * 1e-3),
@@ -377,7 +427,7 @@ def run_fnpu(args):
         line["config"]["decode_share_pct"] = share
         line["config"]["dispatch_trace"] = trace  # [share %, prefill us, decode us] per warm-up step
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(batch, target_seconds=args.ref_seconds)
+        line["cpu_baseline"] = (cpu_baseline_fp8 if args.kv_fp8 else cpu_baseline)(batch, target_seconds=args.ref_seconds)
     elif rank == 0:
         line["cpu_baseline"] = None
     if rank == 0:
@@ -406,6 +456,8 @@ def main(argv=None):
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per attention launch, if measured for this kernel")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kv-fp8", action="store_true",
+                    help="FP8 (e4m3) KV cache; decode-only workloads (qwen_decode)")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)  # at least three untimed warm-up steps
     if args.impl == "reference":

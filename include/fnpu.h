@@ -67,7 +67,31 @@ typedef struct {
     int32_t num_blocks;    /* blocks in the pool */
     int32_t v_in_k_latent; /* 1: MLA latent cache, V aliases K[:, :d_v] */
     float softmax_scale;   /* <= 0 selects 1/sqrt(head_dim_qk) */
+    int32_t kv_fp8;        /* 1: the pools hold the FP8 (e4m3) cache format below; 0: bf16 */
 } fnpu_attn_desc;
+
+/*
+ * FP8 KV cache (kv_fp8 = 1). Decode is bound by KV-cache reads (Sec. 1,
+ * Sec. 3.3); one-byte values halve them. The paper quantises its DeepSeek-R1
+ * deployment to 8 bits (Sec. 4.1) but gives no cache format; this is the
+ * library's. Supported for split K/V with Hkv = 4, d_qk = d_v = 128,
+ * block_size = 16, Hq / Hkv <= 8, and for plans whose sequences are all
+ * one-token decodes; anything else returns FNPU_EUNSUPPORTED.
+ *   Quantisation, per stored row (one slot, one kv head, 128 values):
+ *     scale = amax |x| / 448 in fp32 (1 for a zero row), code = the e4m3 value
+ *     nearest to x / scale (fp32 quotient; ties to the even code; magnitudes
+ *     above 448 saturate to 448; a zero code is stored with a clear sign bit).
+ *     The stored value is value(code) * scale.
+ *   Pools: k_cache and v_cache are byte arrays of num_blocks blocks of 8448
+ *   bytes (16-byte aligned). Within a block, with c = (j mod 8) / 2 and
+ *   r = (j mod 2) + 2 (j / 8) for j in 0..15:
+ *     K: codes [16 slots][4 heads][128], column 16 k + j of a row at byte
+ *        32 c + 4 k + r; then fp32 scales [16 slots][4 heads] at byte 8192
+ *     V: codes [4 heads][128 columns][16 slots], slot j of a column at
+ *        byte 4 c + r; then fp32 scales [16 slots][4 heads] at byte 8192
+ *   The attention products take f16 operands (e4m3 values are exact in f16;
+ *   queries must lie within the f16 range) and fp32 accumulation.
+ */
 
 typedef struct fnpu_plan fnpu_plan; /* opaque, owned by the library */
 
@@ -98,6 +122,8 @@ typedef struct {
  *   k_new, v_new  device bf16 [num_tokens, Hkv, d]; v_new NULL for latent
  *   slot_mapping  device int64 [num_tokens]
  *   k_cache, v_cache  device pools as above; v_cache NULL for latent
+ * With kv_fp8 = 1 each new row is quantised into the FP8 format above (codes
+ * and scale); the result is bit-exact with that definition.
  * Errors: FNPU_EINVAL on NULL pointers or bad shape (nothing launched). A slot
  * >= num_blocks*bs cannot be seen on the host; the kernel skips it and raises
  * the device error flag, reported as FNPU_EDEVICE_RANGE by fnpu_check().
@@ -224,7 +250,8 @@ int fnpu_dispatch_next_share(int32_t share_pct, float prefill_ms, float decode_m
  * Errors: FNPU_EINVAL for bad arguments and for requests whose scratch
  * (4 B per counter, plus 4 B * (Hq/Hkv) * (d + 1) per split, for
  * num_seqs * Hkv * ceil(max_context_len / split_keys) splits) exceeds
- * FNPU_NOALLOC_SCRATCH_BYTES; FNPU_EUNSUPPORTED for other shapes;
+ * FNPU_NOALLOC_SCRATCH_BYTES; FNPU_EUNSUPPORTED for other shapes and for
+ * the FP8 cache (kv_fp8 = 1: plan-based runs only);
  * FNPU_ECUDA. Nothing is launched on error.
  * The first call on a device looks up the scratch array's device address
  * (cudaGetSymbolAddress) while that device is current; make that first call

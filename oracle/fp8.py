@@ -55,7 +55,30 @@ _POS = np.array([e4m3_value(c) for c in range(127)], np.float64)
 
 def e4m3_round(x) -> np.ndarray:
     """Codes of float32 values: nearest e4m3 value, ties to the even code,
-    magnitudes above 448 saturating to 448 (NaN inputs are not expected)."""
+    magnitudes above 448 saturating to 448 (NaN inputs are not expected).
+
+    Per binade: a magnitude a in [2^E, 2^(E+1)) (E >= -6; every a below 2^-6,
+    the subnormals, counts as E = -6) sits on the grid of spacing 2^(E-3)
+    there, so m = a / 2^(E-3) (exact: a power-of-two scaling) rounded half to
+    even is the nearest grid point; it is 8(E+6) + m as a code (code parity =
+    mantissa parity = parity of m, so ties go to the even code, and m = 16
+    carries into the next binade's first code). Equal to the table search
+    ``e4m3_round_by_search`` (a test checks both)."""
+    x = np.asarray(x, np.float32)
+    shape = x.shape
+    x = x.reshape(-1)
+    a = np.minimum(np.abs(x), np.float32(E4M3_MAX))  # every step below is exact in fp32
+    _, e = np.frexp(a)                               # a = f 2^e, f in [0.5, 1); frexp(0) = (0, 0)
+    E = np.maximum(e - 1, -6)
+    E[a < 2.0 ** -6] = -6                            # the subnormals and zero
+    m = np.rint(np.ldexp(a, 3 - E))                  # rint: half to even
+    code = (8 * (E + 6) + m.astype(np.int32)).astype(np.uint8)
+    code[np.signbit(x) & (code != 0)] |= np.uint8(0x80)
+    return code.reshape(shape)
+
+
+def e4m3_round_by_search(x) -> np.ndarray:
+    """The same rounding by search in the table of the 127 finite values."""
     a = np.abs(np.asarray(x, np.float32).astype(np.float64))
     neg = np.signbit(np.asarray(x, np.float32))
     a = np.minimum(a, E4M3_MAX)
@@ -163,8 +186,6 @@ def decode_attention(context_len, block_table, q_bf16, k_pool, v_pool, *, num_q_
     decodes (token s = sequence s at position ctx_s - 1) over the dequantised
     cache: softmax(q k^T * scale) v with k, v = code value * row scale."""
     k_codes, k_scales, v_codes, v_scales = unpack_pools(k_pool, v_pool, num_kv_heads)
-    kd = e4m3_decode(k_codes) * k_scales[..., None].astype(np.float64)
-    vd = e4m3_decode(v_codes) * v_scales[..., None].astype(np.float64)
     g = num_q_heads // num_kv_heads
     sc = scale if scale > 0 else 1.0 / np.sqrt(D)
     qf = bf16_bits_to_f32(q_bf16).astype(np.float64).reshape(-1, num_q_heads, D)
@@ -175,8 +196,9 @@ def decode_attention(context_len, block_table, q_bf16, k_pool, v_pool, *, num_q_
         c = int(context_len[s])
         idx = np.arange(c)
         blk = np.asarray(block_table)[s, idx // BS]
-        keys = kd[blk, idx % BS]     # [c, Hkv, d]
-        vals = vd[blk, idx % BS]
+        # the sequence's keys and values, dequantised: [c, Hkv, d]
+        keys = e4m3_decode(k_codes[blk, idx % BS]) * k_scales[blk, idx % BS][..., None].astype(np.float64)
+        vals = e4m3_decode(v_codes[blk, idx % BS]) * v_scales[blk, idx % BS][..., None].astype(np.float64)
         for h in range(num_q_heads):
             kvh = h // g
             x = keys[:, kvh, :] @ qf[s, h] * sc

@@ -57,7 +57,8 @@ class AttnDesc(ctypes.Structure):
     _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
                 ("head_dim_qk", ctypes.c_int32), ("head_dim_v", ctypes.c_int32),
                 ("block_size", ctypes.c_int32), ("num_blocks", ctypes.c_int32),
-                ("v_in_k_latent", ctypes.c_int32), ("softmax_scale", ctypes.c_float)]
+                ("v_in_k_latent", ctypes.c_int32), ("softmax_scale", ctypes.c_float),
+                ("kv_fp8", ctypes.c_int32)]
 
 
 class PlanOpts(ctypes.Structure):
@@ -149,10 +150,15 @@ def _np(a, dtype) -> np.ndarray:
     return np.ascontiguousarray(np.asarray(a), dtype=dtype)
 
 
+# bytes of one block of the FP8 cache format (16 slots, 4 kv heads, d = 128):
+# K or V codes [16 * 4 * 128] then fp32 scales [16 * 4]
+FP8_BLOCK_BYTES = 16 * 4 * 128 + 16 * 4 * 4
+
+
 def make_desc(num_q_heads, num_kv_heads, head_dim_qk, head_dim_v, block_size, num_blocks,
-              latent=False, softmax_scale=0.0) -> AttnDesc:
+              latent=False, softmax_scale=0.0, kv_fp8=False) -> AttnDesc:
     return AttnDesc(num_q_heads, num_kv_heads, head_dim_qk, head_dim_v, block_size, num_blocks,
-                    int(bool(latent)), float(softmax_scale))
+                    int(bool(latent)), float(softmax_scale), int(bool(kv_fp8)))
 
 
 def kv_append(desc: AttnDesc, k_new, v_new, slot_mapping, k_cache, v_cache, stream=None,

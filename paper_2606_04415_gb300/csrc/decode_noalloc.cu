@@ -299,7 +299,8 @@ extern "C" int fnpu_decode_attn_noalloc(const fnpu_attn_desc *desc, int32_t num_
     const int32_t Hq = desc->num_q_heads, Hkv = desc->num_kv_heads, D = desc->head_dim_qk;
     if (Hq <= 0 || Hkv <= 0 || Hq % Hkv || desc->block_size <= 0 || desc->num_blocks <= 0)
         return FNPU_EINVAL;
-    if (desc->v_in_k_latent || desc->head_dim_v != D || (D != 64 && D != 128) || Hq / Hkv > 8)
+    if (desc->kv_fp8 != 0 && desc->kv_fp8 != 1) return FNPU_EINVAL;
+    if (desc->v_in_k_latent || desc->kv_fp8 || desc->head_dim_v != D || (D != 64 && D != 128) || Hq / Hkv > 8)
         return FNPU_EUNSUPPORTED;
     if (num_seqs == 0) return FNPU_OK;
     if (max_context_len < 1 || split_keys < 0 || (split_keys % 64) != 0) return FNPU_EINVAL;

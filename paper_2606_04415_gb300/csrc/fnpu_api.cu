@@ -242,6 +242,7 @@ bool shape_ok(const fnpu_attn_desc *d, int *status) {
     if (d->num_q_heads <= 0 || d->num_kv_heads <= 0 || d->num_q_heads % d->num_kv_heads) return false;
     if (d->head_dim_qk <= 0 || d->head_dim_v <= 0 || d->block_size <= 0 || d->num_blocks <= 0)
         return false;
+    if (d->kv_fp8 != 0 && d->kv_fp8 != 1) return false;
     if (d->v_in_k_latent) {
         if (d->num_kv_heads != 1 || d->head_dim_v > d->head_dim_qk) return false;
     }
@@ -251,9 +252,17 @@ bool shape_ok(const fnpu_attn_desc *d, int *status) {
     return true;
 }
 
+// The FP8 cache format exists for Hkv = 4, d = 128, 16-slot blocks, G <= 8.
+bool fp8_shape(const fnpu_attn_desc *d) {
+    return !d->v_in_k_latent && decode_fp8_supported(d->head_dim_qk, d->head_dim_v, d->num_kv_heads,
+                                                     d->num_q_heads / d->num_kv_heads, d->block_size);
+}
+
 // Kernels exist for split K/V with d in {64, 128} (decode needs G <= 8) and
 // for the latent layout with d_qk = 576, d_v = 512 and a multiple of 64 heads.
-int kernel_support(const fnpu_attn_desc *d, bool has_decode) {
+// The FP8 cache has a decode kernel only.
+int kernel_support(const fnpu_attn_desc *d, bool has_decode, bool has_prefill) {
+    if (d->kv_fp8) return fp8_shape(d) && !has_prefill ? FNPU_OK : FNPU_EUNSUPPORTED;
     if (d->v_in_k_latent)
         return mla_supported(d->head_dim_qk, d->head_dim_v, d->num_q_heads, d->num_kv_heads) ? FNPU_OK
                                                                                                : FNPU_EUNSUPPORTED;
@@ -302,6 +311,10 @@ int fnpu_kv_append(const fnpu_attn_desc *desc, const void *k_new, const void *v_
                                          reinterpret_cast<uintptr_t>(v_cache)));
     if (mis & 15u) return FNPU_EINVAL;
     if (reinterpret_cast<uintptr_t>(slot_mapping) & 7u) return FNPU_EINVAL;
+    if (desc->kv_fp8) {
+        if (!fp8_shape(desc)) return FNPU_EUNSUPPORTED;
+        return launch_kv_append_fp8(desc, k_new, v_new, slot_mapping, num_tokens, k_cache, v_cache, stream);
+    }
     return launch_kv_append(desc, k_new, v_new, slot_mapping, num_tokens, k_cache, v_cache, stream);
 }
 
@@ -358,10 +371,9 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     }
     if (T > INT32_MAX) return FNPU_EINVAL;
     if (num_seqs > 0) {
-        const int ks = kernel_support(desc, has_decode);
+        const int ks = kernel_support(desc, has_decode, has_prefill);
         if (ks != FNPU_OK) return ks;
     }
-    (void)has_prefill;
 
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return FNPU_ECUDA;
@@ -794,8 +806,9 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
         FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
         return rc;
     }
-    int rc = pl->use_dt ? launch_decode_tma(p, stream, 3 * pl->num_sms)
-                        : launch_decode_mma(p, stream);
+    int rc = pl->desc.kv_fp8 ? launch_decode_fp8(p, stream, 3 * pl->num_sms)
+             : pl->use_dt    ? launch_decode_tma(p, stream, 3 * pl->num_sms)
+                             : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
     return pl->use_tc ? launch_prefill_tc(p, stream, pl->num_sms) : launch_prefill_mma(p, stream);
 }

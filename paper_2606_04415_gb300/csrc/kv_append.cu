@@ -6,6 +6,8 @@
 // thread moves one 16-byte chunk and consecutive threads cover consecutive
 // chunks of the same row: fully coalesced 16-B loads and stores. Pure copy,
 // bit-exact.
+#include <cuda_fp8.h>
+
 #include "common.cuh"
 
 namespace fnpu {
@@ -45,6 +47,93 @@ __global__ void __launch_bounds__(256) kv_append_kernel(
         if (is_k) k_cache[s * k_chunks + c] = v;
         else v_cache[s * v_chunks + cv] = v;
     }
+}
+
+namespace {
+
+// byte position of column `col` of a stored fp8 K row, and of slot `o` of a
+// stored fp8 V column (the four operands of one lane of a 16x8x16 product
+// in four consecutive bytes)
+__device__ __forceinline__ int fp8_kpos(int col) {
+    const int k = col >> 4, j = col & 15;
+    return 32 * ((j & 7) >> 1) + 4 * k + (j & 1) + 2 * (j >> 3);
+}
+__device__ __forceinline__ int fp8_vpos(int o) { return 4 * ((o & 7) >> 1) + (o & 1) + 2 * (o >> 3); }
+
+// two e4m3 codes (low byte first) of two fp32 values, nearest with ties to
+// even, saturating at 448; a zero code is stored positive
+__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
+    uint32_t c = __nv_cvt_float2_to_fp8x2(make_float2(lo, hi), __NV_SATFINITE, __NV_E4M3);
+    if ((c & 0x7Fu) == 0) c &= 0xFF00u;
+    if ((c & 0x7F00u) == 0) c &= 0x00FFu;
+    return c;
+}
+
+constexpr int kF8Hkv = 4, kF8D = 128, kF8Bs = 16;
+constexpr int kF8Codes = kF8Bs * kF8Hkv * kF8D;       // codes of one block (K or V)
+constexpr int kF8Block = kF8Codes + kF8Bs * kF8Hkv * 4;  // + fp32 scales [bs][Hkv]
+
+}  // namespace
+
+// FP8 (e4m3) append, one warp per (token, K or V, kv head) row of 128 values:
+// the row's absolute maximum sets its scale (amax / 448, 1 for a zero row),
+// each value is stored as the code of value / scale. K rows keep the slot-major
+// layout with permuted columns; V rows are scattered into the transposed
+// [head][column][slot] layout. Bit-exact with IEEE fp32 division.
+__global__ void __launch_bounds__(256) kv_append_fp8_kernel(
+    const uint2 *__restrict__ k_new, const uint2 *__restrict__ v_new, const int64_t *__restrict__ slots,
+    int32_t num_tokens, uint8_t *__restrict__ k_pool, uint8_t *__restrict__ v_pool, int64_t num_slots) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nrows = static_cast<int64_t>(num_tokens) * 2 * kF8Hkv;
+    const int64_t step = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+    for (int64_t r = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5; r < nrows; r += step) {
+        const int64_t t = r / (2 * kF8Hkv);
+        const int kv = static_cast<int>(r / kF8Hkv) & 1, h = static_cast<int>(r % kF8Hkv);
+        const uint2 raw = __ldg((kv ? v_new : k_new) + (t * kF8Hkv + h) * (kF8D / 4) + lane);
+        const int64_t s = __ldg(slots + t);
+        if (s < 0) continue;  // warp-uniform: one row per warp
+        if (s >= num_slots) {
+            if (lane == 0 && r % (2 * kF8Hkv) == 0) atomicOr(&g_device_error, 1);
+            continue;
+        }
+        const float x0 = __uint_as_float(raw.x << 16), x1 = __uint_as_float(raw.x & 0xFFFF0000u);
+        const float x2 = __uint_as_float(raw.y << 16), x3 = __uint_as_float(raw.y & 0xFFFF0000u);
+        float a = fmaxf(fmaxf(fabsf(x0), fabsf(x1)), fmaxf(fabsf(x2), fabsf(x3)));
+#pragma unroll
+        for (int m = 16; m > 0; m >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, m));
+        const float scale = a > 0.f ? a / 448.f : 1.f;
+        const uint32_t c01 = e4m3x2(x0 / scale, x1 / scale), c23 = e4m3x2(x2 / scale, x3 / scale);
+        const int o = static_cast<int>(s % kF8Bs);
+        uint8_t *blk = (kv ? v_pool : k_pool) + (s / kF8Bs) * kF8Block;
+        if (kv == 0) {  // columns 4 lane .. 4 lane + 3: two pairs of adjacent bytes
+            uint8_t *row = blk + (o * kF8Hkv + h) * kF8D;
+            *reinterpret_cast<uint16_t *>(row + fp8_kpos(4 * lane)) = static_cast<uint16_t>(c01);
+            *reinterpret_cast<uint16_t *>(row + fp8_kpos(4 * lane + 2)) = static_cast<uint16_t>(c23);
+        } else {
+            uint8_t *col = blk + (h * kF8D + 4 * lane) * kF8Bs + fp8_vpos(o);
+            col[0] = static_cast<uint8_t>(c01);
+            col[kF8Bs] = static_cast<uint8_t>(c01 >> 8);
+            col[2 * kF8Bs] = static_cast<uint8_t>(c23);
+            col[3 * kF8Bs] = static_cast<uint8_t>(c23 >> 8);
+        }
+        if (lane == 0) *reinterpret_cast<float *>(blk + kF8Codes + (o * kF8Hkv + h) * 4) = scale;
+    }
+}
+
+int launch_kv_append_fp8(const fnpu_attn_desc *d, const void *k_new, const void *v_new, const int64_t *slots,
+                         int32_t num_tokens, void *k_cache, void *v_cache, void *stream) {
+    if (num_tokens == 0) return FNPU_OK;
+    const int64_t warps = static_cast<int64_t>(num_tokens) * 2 * kF8Hkv;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (warps + 7) / 8;
+    const int grid = static_cast<int>(want < 32LL * sms ? want : 32LL * sms);
+    kv_append_fp8_kernel<<<grid, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint2 *>(k_new), static_cast<const uint2 *>(v_new), slots, num_tokens,
+        static_cast<uint8_t *>(k_cache), static_cast<uint8_t *>(v_cache),
+        static_cast<int64_t>(d->num_blocks) * kF8Bs);
+    return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
 }
 
 int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_new,

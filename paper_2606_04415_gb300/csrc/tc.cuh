@@ -133,6 +133,15 @@ __device__ __forceinline__ void tma_load_3d_warp(uint32_t dst, const CUtensorMap
         "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
         : "memory");
 }
+// Warp-collective untiled bulk copy global -> shared (both addresses 16-byte
+// aligned, size a multiple of 16), completing on mbarrier `bar`.
+__device__ __forceinline__ void bulk_load_warp(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "{\n .reg .pred p;\n elect.sync _|p, 0xffffffff;\n"
+        " @p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n}\n" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
 __device__ __forceinline__ void mbar_arrive_expect_tx_warp(uint32_t bar, uint32_t bytes) {
     asm volatile(
         "{\n .reg .pred p;\n elect.sync _|p, 0xffffffff;\n"

@@ -5,6 +5,11 @@
 slot mapping and the cache pool), uploads it once as CUDA tensors, builds the
 plan, and runs KV append + attention through the C ABI. Torch provides the
 device memory and the stream; all compute is in the library's kernels.
+
+With ``kv_fp8=True`` the pools hold the library's FP8 (e4m3) cache format
+(byte arrays of ``FP8_BLOCK_BYTES`` per block): they start from the given
+bytes (zeros by default) and the batch's prefix rows enter them through the
+library's quantising append, before the step's own append.
 """
 from __future__ import annotations
 
@@ -12,7 +17,7 @@ from typing import Optional
 
 import numpy as np
 
-from . import (PlanOpts, kv_append, make_desc, mixed_attn_plan, mixed_attn_run)
+from . import (FP8_BLOCK_BYTES, PlanOpts, kv_append, make_desc, mixed_attn_plan, mixed_attn_run)
 
 
 def _to_dev(a: Optional[np.ndarray], torch, dtype, device):
@@ -26,25 +31,53 @@ def _to_dev(a: Optional[np.ndarray], torch, dtype, device):
 
 class DeviceStep:
     def __init__(self, batch, opts: Optional[PlanOpts] = None, device: str = "cuda",
-                 softmax_scale: float = 0.0):
+                 softmax_scale: float = 0.0, kv_fp8: bool = False, pool_init=None):
         import torch
         self.torch = torch
         self.batch = batch
+        self.kv_fp8 = bool(kv_fp8)
         sh = batch.shape
         self.desc = make_desc(sh.num_q_heads, sh.num_kv_heads, sh.head_dim_qk, sh.head_dim_v,
-                              sh.block_size, batch.num_blocks, sh.latent, softmax_scale)
+                              sh.block_size, batch.num_blocks, sh.latent, softmax_scale, kv_fp8)
         bf = torch.bfloat16
         self.q = _to_dev(batch.q, torch, bf, device)
         self.k_new = _to_dev(batch.k_new, torch, bf, device)
         self.v_new = _to_dev(batch.v_new, torch, bf, device)
         self.slot_mapping = _to_dev(batch.slot_mapping, torch, None, device)
-        self.k_cache = _to_dev(batch.k_cache, torch, bf, device)
-        self.v_cache = _to_dev(batch.v_cache, torch, bf, device)
+        if self.kv_fp8:
+            nbytes = batch.num_blocks * FP8_BLOCK_BYTES
+            if pool_init is None:
+                pool_init = (np.zeros(nbytes, np.uint8), np.zeros(nbytes, np.uint8))
+            if pool_init[0].size != nbytes or pool_init[1].size != nbytes:
+                raise ValueError("FP8 pools need num_blocks * FP8_BLOCK_BYTES bytes each")
+            self.k_cache = _to_dev(pool_init[0], torch, None, device)
+            self.v_cache = _to_dev(pool_init[1], torch, None, device)
+            self._fill_prefix(device)
+        else:
+            self.k_cache = _to_dev(batch.k_cache, torch, bf, device)
+            self.v_cache = _to_dev(batch.v_cache, torch, bf, device)
         T = batch.num_tokens
         self.out = torch.empty((T, sh.num_q_heads, sh.head_dim_v), dtype=bf, device=device)
         self.lse = torch.empty((T, sh.num_q_heads), dtype=torch.float32, device=device)
         self.plan = mixed_attn_plan(self.desc, batch.query_len, batch.context_len, batch.phase,
                                     batch.block_table, opts=opts)
+
+    def _fill_prefix(self, device):
+        """Store the batch's prefix rows (its bf16 pool at the prefix slots)
+        through the library's append."""
+        b, sh, torch = self.batch, self.batch.shape, self.torch
+        bs = sh.block_size
+        sl = []
+        for s in range(len(b.query_len)):
+            pos = np.arange(int(b.context_len[s] - b.query_len[s]), dtype=np.int64)
+            sl.append(b.block_table[s, pos // bs].astype(np.int64) * bs + pos % bs)
+        sl = np.concatenate(sl) if sl else np.zeros(0, np.int64)
+        if sl.size == 0:
+            return
+        k = b.k_cache.reshape(-1, sh.num_kv_heads, sh.head_dim_qk)[sl]
+        v = b.v_cache.reshape(-1, sh.num_kv_heads, sh.head_dim_v)[sl]
+        kv_append(self.desc, _to_dev(k, torch, torch.bfloat16, device), _to_dev(v, torch, torch.bfloat16, device),
+                  _to_dev(sl, torch, None, device), self.k_cache, self.v_cache)
 
     def replan(self, opts: Optional[PlanOpts] = None):
         """Plan the same batch again with other options (for instance the
@@ -73,6 +106,8 @@ class DeviceStep:
 
     def cache_bits(self):
         t = self.torch
+        if self.kv_fp8:  # byte pools
+            return self.k_cache.cpu().numpy(), self.v_cache.cpu().numpy()
         kc = self.k_cache.view(t.int16).cpu().numpy().view(np.uint16)
         vc = None if self.v_cache is None else self.v_cache.view(t.int16).cpu().numpy().view(np.uint16)
         return kc, vc

@@ -122,3 +122,29 @@ def test_append_and_run_reject_null_pointers():
     assert lib.fnpu_mixed_attn_run(None, None, None, None, None, None, None) == fnpu.FNPU_EINVAL
     assert lib.fnpu_plan_check(None, None) == fnpu.FNPU_EINVAL
     lib.fnpu_plan_destroy(None)  # ignored
+
+
+def test_fp8_cache_validation():
+    """The FP8 cache: kv_fp8 outside {0, 1} is invalid; other shapes, latent
+    caches and plans with prefill work are unsupported; all decided on the
+    host before any CUDA call."""
+    lib = fnpu.load()
+    bt = np.zeros((2, 4), np.int32)
+    bad = fnpu.make_desc(**QWEN)
+    bad.kv_fp8 = 2
+    assert _plan_rc(bad, [1], [5], [1], bt[:1]) == fnpu.FNPU_EINVAL
+    assert lib.fnpu_kv_append(ctypes.byref(bad), 16, 32, 64, 4, 128, 256, None) == fnpu.FNPU_EINVAL
+    fp8 = fnpu.make_desc(**QWEN, kv_fp8=True)
+    assert _plan_rc(fp8, [8, 1], [8, 20], [0, 1], bt) == fnpu.FNPU_EUNSUPPORTED      # prefill chunk
+    assert _plan_rc(fp8, [3], [20], [1], bt[:1]) == fnpu.FNPU_EUNSUPPORTED          # multi-token decode
+    for other in (dict(head_dim_qk=64, head_dim_v=64), dict(num_kv_heads=2, num_q_heads=14),
+                  dict(block_size=32), dict(num_q_heads=36)):
+        d = fnpu.make_desc(**dict(QWEN, **other), kv_fp8=True)
+        assert _plan_rc(d, [1], [5], [1], bt[:1]) == fnpu.FNPU_EUNSUPPORTED, other
+        assert lib.fnpu_kv_append(ctypes.byref(d), 16, 32, 64, 4, 128, 256, None) == fnpu.FNPU_EUNSUPPORTED
+    lat = fnpu.make_desc(128, 1, 576, 512, 64, 8, latent=True, kv_fp8=True)
+    assert _plan_rc(lat, [1], [5], [1], bt[:1]) == fnpu.FNPU_EUNSUPPORTED
+    # the allocation-free decode entry point takes bf16 caches only
+    rc = lib.fnpu_decode_attn_noalloc(ctypes.byref(fp8), 1, 16, 32, 4, 5, 0, 48, 64, 80, 96, 112, None)
+    assert rc == fnpu.FNPU_EUNSUPPORTED
+    assert fnpu.FP8_BLOCK_BYTES == 8448

@@ -139,3 +139,16 @@ def test_matches_the_bf16_oracle_when_every_scale_is_one():
     ref_o, ref_l = oracle.attention(np.ones(3, np.int32), ctx, bt, q, kdq, vdq, num_q_heads=hq,
                                     num_kv_heads=hkv, head_dim_qk=128, head_dim_v=128, block_size=16)
     assert np.abs(out - ref_o).max() < 1e-12 and np.abs(lse - ref_l).max() < 1e-12
+
+
+def test_binade_rounding_equals_the_table_search():
+    """The per-binade rounding and the table search agree on random
+    magnitudes over the whole range, on every value, and on every midpoint
+    between neighbouring values (the ties)."""
+    rng = np.random.default_rng(7)
+    x = (rng.standard_normal(200000) * np.exp2(rng.uniform(-14, 10, 200000))).astype(np.float32)
+    vals = np.array([fp8.e4m3_value(c) for c in range(127)])
+    mids = ((vals[1:] + vals[:-1]) / 2).astype(np.float32)
+    near = np.concatenate([np.nextafter(mids, np.float32(0)), np.nextafter(mids, np.float32(1e9))])
+    for arr in (x, vals.astype(np.float32), mids, -mids, near, np.array([0, -0.0, 448, 449, 470, 1e38], np.float32)):
+        assert np.array_equal(fp8.e4m3_round(arr), fp8.e4m3_round_by_search(arr))

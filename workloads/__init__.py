@@ -260,6 +260,35 @@ def make_batch(name: str, seed: int = 0) -> Batch:
     return build_batch(shape, q, ctx, ph, rng, name=name, seed=seed, num_blocks=nb)
 
 
+def prefix_slots(batch: Batch) -> np.ndarray:
+    """Slots of every sequence's prefix positions (< ctx - q), sequence by
+    sequence: the rows that are in the cache before the step."""
+    bs = batch.shape.block_size
+    out = []
+    for s in range(batch.num_seqs):
+        pos = np.arange(int(batch.context_len[s] - batch.query_len[s]), dtype=np.int64)
+        out.append(batch.block_table[s, pos // bs].astype(np.int64) * bs + pos % bs)
+    return np.concatenate(out) if out else np.zeros(0, np.int64)
+
+
+def prefix_rows(batch: Batch) -> tuple:
+    """(k_rows, v_rows, slots): the bf16 bits of the prefix rows of the pool,
+    for filling a cache of another storage format through its own append."""
+    sl = prefix_slots(batch)
+    sh = batch.shape
+    k = batch.k_cache.reshape(-1, sh.num_kv_heads, sh.head_dim_qk)[sl]
+    v = batch.v_cache.reshape(-1, sh.num_kv_heads, sh.head_dim_v)[sl]
+    return np.ascontiguousarray(k), np.ascontiguousarray(v), sl
+
+
+def stale_pool_bytes(nbytes: int, seed: int) -> tuple:
+    """Seeded random bytes for the K and V pools of a byte-format cache before
+    any append: every byte value occurs, NaN codes and NaN scales included, so a
+    kernel that reads a slot it must not see goes wrong visibly."""
+    rng = np.random.default_rng([seed, 0xF8])
+    return (rng.integers(0, 256, nbytes, dtype=np.uint8), rng.integers(0, 256, nbytes, dtype=np.uint8))
+
+
 def pairs(batch: Batch) -> int:
     """Visible (query, key) pairs: sum over seqs of q*p + q(q+1)/2."""
     q = batch.query_len.astype(np.int64)
@@ -267,8 +296,12 @@ def pairs(batch: Batch) -> int:
     return int((q * p + q * (q + 1) // 2).sum())
 
 
-def algorithmic_work(batch: Batch) -> dict:
+def algorithmic_work(batch: Batch, kv_fp8: bool = False) -> dict:
     """Algorithmic FLOPs and HBM bytes of one step (append + attention).
+
+    With kv_fp8 the cache rows are one-byte codes plus one fp32 scale per
+    (slot, kv head) row of K and of V; the append reads bf16 rows and writes
+    that format.
 
     FLOPs count QK^T and PV over visible pairs only: 2*Hq*pairs*(d_qk + d_v).
     Bytes count each cache row of every sequence read once, Q read, O (bf16)
@@ -281,11 +314,14 @@ def algorithmic_work(batch: Batch) -> dict:
     ctx = batch.context_len.astype(np.int64)
     flops = 2 * sh.num_q_heads * pairs(batch) * (sh.head_dim_qk + sh.head_dim_v)
     row_bytes = 2 * (sh.head_dim_qk if sh.latent else sh.num_kv_heads * (sh.head_dim_qk + sh.head_dim_v))
-    kv_read = int(ctx.sum()) * row_bytes
+    cache_row = row_bytes
+    if kv_fp8:
+        cache_row = sh.num_kv_heads * (sh.head_dim_qk + 4 + sh.head_dim_v + 4)
+    kv_read = int(ctx.sum()) * cache_row
     q_read = T * sh.num_q_heads * sh.head_dim_qk * 2
     o_write = T * sh.num_q_heads * sh.head_dim_v * 2
     lse_write = T * sh.num_q_heads * 4
-    append = 2 * T * row_bytes
+    append = T * (row_bytes + cache_row)
     meta = 8 * T + 4 * int(((ctx + sh.block_size - 1) // sh.block_size).sum())
     return {
         "flops": int(flops),
