@@ -13,8 +13,9 @@
 // split-merge kernel after it). What differs:
 //   * A 16-key stage is one block: a 4-D box of K codes lands head-major
 //     (slot dimension listed before the head dimension, 128-byte swizzle),
-//     a 4-D box of V codes lands [head][column][16 slots], and two 256-byte
-//     bulk copies bring the block's K and V scales.
+//     one bulk copy brings the block's V codes ([head][column][16 slots]) with
+//     the V scales behind them, and another the K scales (a tensor box of
+//     the V codes would be 512 rows of 16 bytes; the bulk copy is one request).
 //   * The products run in f16: e4m3 values are exact in f16, the query is
 //     converted once per item, and the codes go through cvt e4m3x2 -> f16x2.
 //     The column permutation of K puts the four values a lane needs for one
@@ -58,7 +59,7 @@ constexpr int kSmemBytes = kBarOff + 8 * kNumBars + 32;  // + item ring [4] and 
 static_assert(kCodeBytes % 1024 == 0 && kStageStride % 1024 == 0, "swizzle atoms");
 
 struct Fp8Maps {
-    CUtensorMap k, v;
+    CUtensorMap k;
 };
 
 struct DtGeo {
@@ -68,10 +69,13 @@ struct DtGeo {
     int split, ns, part_base, group;
 };
 
-// e4m3 pair (low byte first) -> f16x2 (low half first)
-__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two) {
-    const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2(static_cast<__nv_fp8x2_storage_t>(two & 0xFFFFu), __NV_E4M3);
-    return static_cast<uint32_t>(h.x) | (static_cast<uint32_t>(h.y) << 16);
+// four e4m3 codes (bytes 0..3 of w) -> two f16x2: lo = (byte 0, byte 1),
+// hi = (byte 2, byte 3), the lower byte in the lower half
+__device__ __forceinline__ void e4m3x4_to_f16x2x2(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    asm("{\n .reg .b16 l, h;\n mov.b32 {l, h}, %2;\n cvt.rn.f16x2.e4m3x2 %0, l;\n"
+        " cvt.rn.f16x2.e4m3x2 %1, h;\n}\n"
+        : "=r"(lo), "=r"(hi)
+        : "r"(w));
 }
 
 __device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t b) {
@@ -147,7 +151,6 @@ __global__ void __launch_bounds__(kThreads, 3)
     }
     if (warp == kWarps && lane == 0) {
         tc::prefetch_tmap(&maps.k);
-        tc::prefetch_tmap(&maps.v);
     }
     __syncthreads();
 
@@ -188,13 +191,14 @@ __global__ void __launch_bounds__(kThreads, 3)
         const int rel = key0 / kKeys - g.kb / kKeys;
         int blk = __shfl_sync(0xffffffffu, blk_lane, rel & 31);
         if (rel >= 32) blk = __ldg(p.block_table + static_cast<int64_t>(g.bt_row) * p.bt_stride + key0 / kKeys);
-        const uint32_t sK = s_base + st * kStageStride, sV = sK + kCodeBytes, sS = sV + kCodeBytes;
+        // stage: K codes (head-major, swizzled) | V codes and V scales (the
+        // block's V half as stored: one contiguous copy) | K scales
+        const uint32_t sK = s_base + st * kStageStride, sV = sK + kCodeBytes;
+        const int64_t boff = static_cast<int64_t>(blk) * kBlockBytes;
         tc::mbar_arrive_expect_tx_warp(FULL(st), kStageBytes);
         tc::tma_load_4d_warp(sK, &maps.k, FULL(st), 0, 0, 0, blk);
-        tc::tma_load_4d_warp(sV, &maps.v, FULL(st), 0, 0, 0, blk);
-        const int64_t boff = static_cast<int64_t>(blk) * kBlockBytes + kCodeBytes;
-        tc::bulk_load_warp(sS, k_pool + boff, kScaleBytes, FULL(st));
-        tc::bulk_load_warp(sS + kScaleBytes, v_pool + boff, kScaleBytes, FULL(st));
+        tc::bulk_load_warp(sV, v_pool + boff, kBlockBytes, FULL(st));
+        tc::bulk_load_warp(sV + kBlockBytes, k_pool + boff + kCodeBytes, kScaleBytes, FULL(st));
         return true;
     };
 
@@ -268,7 +272,9 @@ __global__ void __launch_bounds__(kThreads, 3)
 #pragma unroll
             for (int mt = 0; mt < kD / 16; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
             float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-            float vm = 0.f;  // running max of the item's V scales: o holds O^T / vm
+            // vm: a power of two at or above every V scale of the item so far;
+            // o holds O^T / vm
+            float vm = 0.f;
             const int nkeys = cur.ke - cur.kb;
             for (int i = 0; i < ntiles; ++i) {
                 const int gs = g + i;
@@ -280,8 +286,8 @@ __global__ void __launch_bounds__(kThreads, 3)
                     if (has_next) nit = p.ditems[idx_n];
                 }
                 const uint8_t *tK = smem + st * kStageStride, *tV = tK + kCodeBytes;
-                const float *kscale = reinterpret_cast<const float *>(tV + kCodeBytes);
-                const float *vscale = kscale + kKeys * kHkv;
+                const float *vscale = reinterpret_cast<const float *>(tV + kCodeBytes);
+                const float *kscale = vscale + kKeys * kHkv;
                 const int nv = nkeys - i * kKeys;  // valid keys in this stage (>= 1)
                 const bool v0 = g8 < nv, v1 = g8 + 8 < nv;
                 // S^T (keys x query heads): rows g8 and g8 + 8 of this head's K codes,
@@ -298,31 +304,47 @@ __global__ void __launch_bounds__(kThreads, 3)
                 float s[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
-                    const uint32_t a0 = e4m3x2_to_f16x2(kw0[kk]), a2 = e4m3x2_to_f16x2(kw0[kk] >> 16);
-                    const uint32_t a1 = e4m3x2_to_f16x2(kw1[kk]), a3 = e4m3x2_to_f16x2(kw1[kk] >> 16);
+                    uint32_t a0, a1, a2, a3;
+                    e4m3x4_to_f16x2x2(kw0[kk], a0, a2);
+                    e4m3x4_to_f16x2x2(kw1[kk], a1, a3);
                     mma_f16_16816(s, a0, a1, a2, a3, qb[kk][0], qb[kk][1]);
                 }
-                const float ks0 = v0 ? kscale[g8 * kHkv + head] : 0.f;
-                const float ks1 = v1 ? kscale[(g8 + 8) * kHkv + head] : 0.f;
-                const float x0 = v0 ? s[0] * ks0 * p.scale_log2 : -INFINITY;
-                const float x1 = v0 ? s[1] * ks0 * p.scale_log2 : -INFINITY;
-                const float x2 = v1 ? s[2] * ks1 * p.scale_log2 : -INFINITY;
-                const float x3 = v1 ? s[3] * ks1 * p.scale_log2 : -INFINITY;
-                float t0 = fmaxf(x0, x2), t1 = fmaxf(x1, x3);
-                t0 = warp_max_xor(t0, 4); t0 = warp_max_xor(t0, 8); t0 = warp_max_xor(t0, 16);
-                t1 = warp_max_xor(t1, 4); t1 = warp_max_xor(t1, 8); t1 = warp_max_xor(t1, 16);
+                // V^T operands (keys 2c, 2c + 1, 2c + 8, 2c + 9 of columns 16 mt + g8
+                // and + 8): loaded now, converted after the softmax
+                uint32_t vw0[kD / 16], vw1[kD / 16];
+#pragma unroll
+                for (int mt = 0; mt < kD / 16; ++mt) {
+                    vw0[mt] = *reinterpret_cast<const uint32_t *>(tV + (head * kD + 16 * mt + g8) * kKeys + 4 * c);
+                    vw1[mt] = *reinterpret_cast<const uint32_t *>(tV + (head * kD + 16 * mt + g8 + 8) * kKeys + 4 * c);
+                }
+                const float ks0 = v0 ? kscale[g8 * kHkv + head] * p.scale_log2 : 0.f;
+                const float ks1 = v1 ? kscale[(g8 + 8) * kHkv + head] * p.scale_log2 : 0.f;
+                const float vs0 = v0 ? vscale[g8 * kHkv + head] : 0.f;
+                const float vs1 = v1 ? vscale[(g8 + 8) * kHkv + head] : 0.f;
+                const float x0 = v0 ? s[0] * ks0 : -INFINITY;
+                const float x1 = v0 ? s[1] * ks0 : -INFINITY;
+                const float x2 = v1 ? s[2] * ks1 : -INFINITY;
+                const float x3 = v1 ? s[3] * ks1 : -INFINITY;
+                float t0 = fmaxf(x0, x2), t1 = fmaxf(x1, x3), vt = fmaxf(vs0, vs1);
+                t0 = warp_max_xor(t0, 4); t1 = warp_max_xor(t1, 4); vt = warp_max_xor(vt, 4);
+                t0 = warp_max_xor(t0, 8); t1 = warp_max_xor(t1, 8); vt = warp_max_xor(vt, 8);
+                t0 = warp_max_xor(t0, 16); t1 = warp_max_xor(t1, 16); vt = warp_max_xor(vt, 16);
                 const float mn0 = fmaxf(m0, t0), mn1 = fmaxf(m1, t1);
                 const float b0 = (mn0 == -INFINITY) ? 0.f : mn0;
                 const float b1 = (mn1 == -INFINITY) ? 0.f : mn1;
-                // the V scales of this stage's keys; probabilities enter P V as
-                // p * vs / vm (at most 1, so f16 keeps their precision)
-                const float vs0 = v0 ? vscale[g8 * kHkv + head] : 0.f;
-                const float vs1 = v1 ? vscale[(g8 + 8) * kHkv + head] : 0.f;
-                float vt = fmaxf(vs0, vs1);
-                vt = warp_max_xor(vt, 4); vt = warp_max_xor(vt, 8); vt = warp_max_xor(vt, 16);
-                const float vmn = fmaxf(vm, vt);  // > 0: key 0 of a stage is valid, its scale positive
-                const float rv = __fdividef(vm, vmn), ivm = 1.f / vmn;
-                vm = vmn;
+                // probabilities enter P V as p * vs / vm, at most 1, so that f16
+                // keeps their precision. vt > 0 (key 0 of a stage is valid, scales
+                // are positive) and warp-uniform; vm grows to the power of two at
+                // or above it, so 1 / vm and the rescale vm_old / vm_new are exact.
+                float rv = 1.f;
+                if (vt > vm) {
+                    const uint32_t bits = __float_as_uint(vt);
+                    const uint32_t up = (bits & 0x7FFFFFu) ? (bits & 0x7F800000u) + 0x800000u : bits;
+                    const float vmn = bits < 0x800000u ? 1.17549435e-38f : __uint_as_float(up);  // subnormal: 2^-126
+                    rv = vm * __uint_as_float(0x7F000000u - __float_as_uint(vmn));
+                    vm = vmn;
+                }
+                const float ivm = __uint_as_float(0x7F000000u - __float_as_uint(vm));  // 2^-e for vm = 2^e
                 const float al0 = fast_exp2(m0 - b0), al1 = fast_exp2(m1 - b1);
                 const float ro0 = al0 * rv, ro1 = al1 * rv;
                 const float p0 = fast_exp2(x0 - b0), p1 = fast_exp2(x1 - b1);
@@ -331,25 +353,34 @@ __global__ void __launch_bounds__(kThreads, 3)
                 l1 = l1 * al1 + p1 + p3;
                 m0 = mn0;
                 m1 = mn1;
+                if (__any_sync(0xffffffffu, (ro0 != 1.f) | (ro1 != 1.f))) {  // most stages move neither maximum
 #pragma unroll
-                for (int mt = 0; mt < kD / 16; ++mt) {
-                    o[mt][0] *= ro0; o[mt][1] *= ro1; o[mt][2] *= ro0; o[mt][3] *= ro1;
+                    for (int mt = 0; mt < kD / 16; ++mt) {
+                        o[mt][0] *= ro0; o[mt][1] *= ro1; o[mt][2] *= ro0; o[mt][3] *= ro1;
+                    }
                 }
                 // probabilities times the V scale of their key over vm (0 past the item)
                 const float w0 = vs0 * ivm, w1 = vs1 * ivm;
                 const uint32_t pb0 = movmatrix_trans(pack_f16x2(p0 * w0, p1 * w0));
                 const uint32_t pb1 = movmatrix_trans(pack_f16x2(p2 * w1, p3 * w1));
-                // V^T operands: keys 2c, 2c + 1, 2c + 8, 2c + 9 of columns 16 mt + g8
-                // (+ 8), zero for keys past the item
-                const uint32_t lo_keep = (2 * c < nv ? 0x0000FFFFu : 0u) | (2 * c + 1 < nv ? 0xFFFF0000u : 0u);
-                const uint32_t hi_keep = (2 * c + 8 < nv ? 0x0000FFFFu : 0u) | (2 * c + 9 < nv ? 0xFFFF0000u : 0u);
+                if (nv >= kKeys) {
 #pragma unroll
-                for (int mt = 0; mt < kD / 16; ++mt) {
-                    const uint32_t w0 = *reinterpret_cast<const uint32_t *>(tV + (head * kD + 16 * mt + g8) * kKeys + 4 * c);
-                    const uint32_t w1 = *reinterpret_cast<const uint32_t *>(tV + (head * kD + 16 * mt + g8 + 8) * kKeys + 4 * c);
-                    const uint32_t a0 = e4m3x2_to_f16x2(w0) & lo_keep, a2 = e4m3x2_to_f16x2(w0 >> 16) & hi_keep;
-                    const uint32_t a1 = e4m3x2_to_f16x2(w1) & lo_keep, a3 = e4m3x2_to_f16x2(w1 >> 16) & hi_keep;
-                    mma_f16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+                    for (int mt = 0; mt < kD / 16; ++mt) {
+                        uint32_t a0, a1, a2, a3;
+                        e4m3x4_to_f16x2x2(vw0[mt], a0, a2);
+                        e4m3x4_to_f16x2x2(vw1[mt], a1, a3);
+                        mma_f16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+                    }
+                } else {  // the item's last, partial block: V of keys past it set to zero
+                    const uint32_t lo_keep = (2 * c < nv ? 0x0000FFFFu : 0u) | (2 * c + 1 < nv ? 0xFFFF0000u : 0u);
+                    const uint32_t hi_keep = (2 * c + 8 < nv ? 0x0000FFFFu : 0u) | (2 * c + 9 < nv ? 0xFFFF0000u : 0u);
+#pragma unroll
+                    for (int mt = 0; mt < kD / 16; ++mt) {
+                        uint32_t a0, a1, a2, a3;
+                        e4m3x4_to_f16x2x2(vw0[mt], a0, a2);
+                        e4m3x4_to_f16x2x2(vw1[mt], a1, a3);
+                        mma_f16_16816(o[mt], a0 & lo_keep, a1 & lo_keep, a2 & hi_keep, a3 & hi_keep, pb0, pb1);
+                    }
                 }
                 __syncwarp();
                 tc::mbar_arrive_warp(EMPTY(st));
@@ -463,19 +494,6 @@ bool encode_k_map(CUtensorMap *m, const void *base, int nblocks) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// V codes: bytes [block][head][128 columns][16 slots]; a box is one block.
-bool encode_v_map(CUtensorMap *m, const void *base, int nblocks) {
-    EncodeTiledFn enc = fp8_encoder();
-    if (!enc) return false;
-    cuuint64_t dims[4] = {kKeys, static_cast<cuuint64_t>(kD), kHkv, static_cast<cuuint64_t>(nblocks)};
-    cuuint64_t strides[3] = {kKeys, kKeys * kD, kBlockBytes};
-    cuuint32_t box[4] = {kKeys, kD, kHkv, 1};
-    cuuint32_t es[4] = {1, 1, 1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void *>(base), dims, strides, box, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 }  // namespace
 
 bool decode_fp8_supported(int d_qk, int d_v, int hkv, int group, int block_size) {
@@ -486,7 +504,7 @@ int launch_decode_fp8(const AttnParams &p, void *stream, int max_ctas) {
     if (p.num_ditems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     Fp8Maps maps;
-    if (!encode_k_map(&maps.k, p.k_cache, p.num_blocks) || !encode_v_map(&maps.v, p.v_cache, p.num_blocks))
+    if (!encode_k_map(&maps.k, p.k_cache, p.num_blocks))
         return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled (fp8 decode)");
     FNPU_CUDA_TRY(cudaFuncSetAttribute(decode_fp8_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes));
     const int grid = p.num_ditems < max_ctas ? p.num_ditems : max_ctas;
