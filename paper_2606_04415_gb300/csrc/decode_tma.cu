@@ -7,11 +7,13 @@
 // memory for d = 128 -- so that three CTAs share an SM and a few SMs alone
 // can stream decode work while the others run prefill (Sec. 3.4).
 //   * Persistent CTAs take items -- a sequence's key range, longest first --
-//     from an atomic queue one item ahead of use (the last CTA out resets it);
-//     the next item's descriptor, block ids and query are loaded during the
-//     current item, so an item boundary costs no memory round trip. (Taking
-//     two items ahead left CTAs idle when items were few: the first CTAs
-//     reserved them all.)
+//     CTA b item b first, then from an atomic queue one item ahead of use (the
+//     last CTA out resets it); the next item's descriptor, block ids and
+//     query are loaded during the current item, so an item boundary costs no
+//     memory round trip, and a descriptor carries the item's query token,
+//     block-table row and first four block ids, so that a CTA issues its
+//     first copies one load after it starts. (Taking two items ahead left
+//     CTAs idle when items were few: the first CTAs reserved them all.)
 //   * A 2-stage ring of 16-key stages holds K and V of all four kv heads. A
 //     producer warp issues the TMA copies (four boxes of 16 slots x 4 heads x
 //     64 columns for d = 128) as soon as a stage is free; issuing them from a
@@ -76,6 +78,7 @@ struct DtGeo {
     int bt_row;
     int kb, ke;     // keys [kb, ke)
     int split, ns, part_base, group;
+    int b0, b1, b2, b3;  // ids of the item's first four blocks
 };
 
 template <int D>
@@ -126,7 +129,7 @@ __global__ void __launch_bounds__(kThreads, 3)
             tc::mbar_init(FULL(s), 1);
             tc::mbar_init(EMPTY(s), kWarps);
         }
-        ring[0] = atomicAdd(sched, 1);
+        ring[0] = blockIdx.x;  // the first item without the queue (grid <= items); the queue serves the rest
         *abort_flag = 0;
         tc::fence_mbar_init();
     }
@@ -144,10 +147,14 @@ __global__ void __launch_bounds__(kThreads, 3)
         atomicOr(p.err, 1);
         return false;
     };
-    auto geo_of = [&](const DecodeItem &it, const SeqInfo &si) {
+    auto geo_of = [&](const DecodeItem &it) {
         DtGeo g;
-        g.t = si.q_start;
-        g.bt_row = si.bt_row;
+        g.t = it.q_start;
+        g.bt_row = it.bt_row;
+        g.b0 = it.blk[0];
+        g.b1 = it.blk[1];
+        g.b2 = it.blk[2];
+        g.b3 = it.blk[3];
         g.kb = it.key_begin;
         g.ke = it.key_end;
         g.split = it.split;
@@ -170,9 +177,14 @@ __global__ void __launch_bounds__(kThreads, 3)
         const int st = gs % kStages;
         if (gs >= kStages && !wait(EMPTY(st), ((gs / kStages) - 1) & 1)) return false;
         const int key0 = g.kb + j * kKeys;
-        const int rel = key0 / bs - g.kb / bs;
-        int blk = __shfl_sync(0xffffffffu, blk_lane, rel & 31);
-        if (rel >= 32) blk = __ldg(p.block_table + static_cast<int64_t>(g.bt_row) * p.bt_stride + key0 / bs);
+        const int rel = key0 / bs - g.kb / bs;  // warp-uniform
+        int blk;
+        if (rel < 4) {  // from the item itself: the lanes' block-id loads may still be in flight
+            blk = rel == 0 ? g.b0 : rel == 1 ? g.b1 : rel == 2 ? g.b2 : g.b3;
+        } else {
+            blk = __shfl_sync(0xffffffffu, blk_lane, rel & 31);
+            if (rel >= 32) blk = __ldg(p.block_table + static_cast<int64_t>(g.bt_row) * p.bt_stride + key0 / bs);
+        }
         const uint32_t sK = s_base + st * Cfg::kStageBytes, sV = sK + Cfg::kTileBytes;
         tc::mbar_arrive_expect_tx_warp(FULL(st), Cfg::kStageBytes);
 #pragma unroll
@@ -190,28 +202,24 @@ __global__ void __launch_bounds__(kThreads, 3)
         // ahead, so that the queue still balances the CTAs), publishes its
         // index in the item ring before it issues stage 2 of the current item
         // (the compute warps read it after that stage has landed), and loads
-        // the next item's descriptor, sequence row and block ids one stage
-        // apart, so that no dependent memory round trip sits between stages.
+        // the next item's descriptor, then a stage later its block ids, so
+        // that no dependent memory round trip sits between stages. An item's
+        // first four blocks come with its descriptor.
         int gs = 0;
         bool ok = true;
         int idx = ring[0];
         DecodeItem it{};
-        SeqInfo si{};
-        if (idx < n_items) {
-            it = p.ditems[idx];
-            si = p.seqs[it.seq];
-        }
-        DtGeo cur = geo_of(it, si);
+        if (idx < n_items) it = p.ditems[idx];
+        DtGeo cur = geo_of(it);
         int blk_lane = idx < n_items ? load_blk_lane(p, cur, lane) : 0;
         for (int k = 0; ok && idx < n_items; ++k) {
             int a = 0;
-            if (lane == 0) a = atomicAdd(sched, 1);  // the next item
+            if (lane == 0) a = static_cast<int>(gridDim.x) + atomicAdd(sched, 1);  // the next item
             const int ntiles = (cur.ke - cur.kb + kKeys - 1) / kKeys;
             const int spub = ntiles > 2 ? 2 : ntiles - 1;
-            const int s1 = spub + 1 < ntiles ? spub + 1 : spub, s2 = spub + 2 < ntiles ? spub + 2 : s1;
+            const int s1 = spub + 1 < ntiles ? spub + 1 : spub;
             int idx_n = n_items;
             DecodeItem nit{};
-            SeqInfo nsi{};
             DtGeo nxt{};
             int blk_lane_n = 0;
             for (int i = 0; i < ntiles; ++i, ++gs) {
@@ -222,9 +230,8 @@ __global__ void __launch_bounds__(kThreads, 3)
                     if (idx_n < n_items) nit = p.ditems[idx_n];
                 }
                 if (!issue(cur, i, blk_lane, gs)) { ok = false; break; }
-                if (idx_n < n_items && i == s1) nsi = p.seqs[nit.seq];
-                if (idx_n < n_items && i == s2) {
-                    nxt = geo_of(nit, nsi);
+                if (idx_n < n_items && i == s1) {
+                    nxt = geo_of(nit);
                     blk_lane_n = load_blk_lane(p, nxt, lane);
                 }
             }
@@ -237,8 +244,7 @@ __global__ void __launch_bounds__(kThreads, 3)
         int idx = ring[0];
         DtGeo cur;
         {
-            const DecodeItem it = p.ditems[idx];
-            cur = geo_of(it, p.seqs[it.seq]);
+            cur = geo_of(p.ditems[idx]);
         }
         uint32_t qb[D / 16][2];
         load_q<D>(p, cur.t, head, g8, c, qb);
@@ -250,7 +256,6 @@ __global__ void __launch_bounds__(kThreads, 3)
             int idx_n = n_items;
             bool has_next = false;
             DecodeItem nit{};
-            SeqInfo nsi{};
             DtGeo nxt{};
             uint32_t qn[D / 16][2];
 
@@ -320,11 +325,10 @@ __global__ void __launch_bounds__(kThreads, 3)
                 if (tail) tc::fence_proxy_async_smem();  // order the zeroing before the next TMA write
                 __syncwarp();
                 tc::mbar_arrive_warp(EMPTY(st));
-                // the next item: its sequence row after this stage, its query a
-                // stage later (at once for a short item)
-                if (has_next && i == spub) nsi = p.seqs[nit.seq];
+                // the next item's query: a stage after its descriptor (at once for
+                // a short item)
                 if (has_next && i == (spub + 1 < ntiles ? spub + 1 : spub)) {
-                    nxt = geo_of(nit, nsi);
+                    nxt = geo_of(nit);
                     load_q<D>(p, nxt.t, head, g8, c, qn);
                 }
             }

@@ -416,6 +416,14 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     // with 128. The per-head kernel aims at about 3 waves of 2 CTAs per SM.
     // the queue a sequence's work enters: decode items for one-token decodes
     auto decode_queue = [&](int32_t s) { return phase[s] == 1 && query_len[s] == 1; };
+    // a decode item with its sequence's fields and its first four block ids
+    auto decode_item = [&](int32_t s, int32_t kvh, int32_t kb, int32_t ke, int32_t sp, int32_t ns, int32_t base,
+                           int32_t grp) {
+        DecodeItem it{s, kvh, kb, ke, sp, ns, base, grp, seqs[s].q_start, seqs[s].bt_row, 0, 0, {0, 0, 0, 0}};
+        for (int32_t i = 0; i < 4 && kb / bs + i <= (ke - 1) / bs; ++i)
+            it.blk[i] = block_table[static_cast<int64_t>(s) * block_table_stride + kb / bs + i];
+        return it;
+    };
     int64_t dec_keys = 0;
     for (int32_t s = 0; s < num_seqs; ++s)
         if (decode_queue(s))
@@ -508,7 +516,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
             }
             for (int32_t sp = 0; sp < ns; ++sp) {
                 const int32_t kb = sp * sk, ke = std::min(c, kb + sk);
-                ditems.push_back(DecodeItem{s, 0, kb, ke, sp, ns, base, 0});
+                ditems.push_back(decode_item(s, 0, kb, ke, sp, ns, base, 0));
             }
         } else if (decode_queue(s)) {
             const int32_t ns = (c + split - 1) / split;
@@ -518,7 +526,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                 if (ns > 1) parts += ns;
                 for (int32_t sp = 0; sp < ns; ++sp) {
                     const int32_t kb = sp * split, ke = std::min(c, kb + split);
-                    ditems.push_back(DecodeItem{s, kvh, kb, ke, sp, ns, base, grp});
+                    ditems.push_back(decode_item(s, kvh, kb, ke, sp, ns, base, grp));
                 }
             }
         } else if (pl->use_tc) {

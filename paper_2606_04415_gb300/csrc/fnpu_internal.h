@@ -12,12 +12,16 @@ namespace fnpu {
 // sequence's single query position, for kv head `kvh` and its G query heads
 // (per-head kernel) or for every kv head (all-heads kernel, kvh = 0). Splits
 // of one group share `group` (their merge counter) and write partial results
-// to scratch rows part_base + split.
+// to scratch rows part_base + split. The item also carries its sequence's
+// query token and block-table row and the ids of its first four blocks, so
+// that a kernel can issue its first copies after one load.
 struct DecodeItem {
     int32_t seq, kvh, key_begin, key_end;
     int32_t split, num_splits, part_base, group;
+    int32_t q_start, bt_row, pad0, pad1;
+    int32_t blk[4];  // block_table[bt_row][key_begin / bs + i], 0 past the item
 };
-static_assert(sizeof(DecodeItem) == 32, "DecodeItem layout");
+static_assert(sizeof(DecodeItem) == 64, "DecodeItem layout");
 
 // One prefill tile: query rows [row_begin, row_begin + rows) of sequence
 // `seq`'s chunk for query head `head` (the mma.sync path) or for kv head

@@ -376,17 +376,33 @@ def test_mla_long_decode_many_pieces():
     _compare(batch, out, lse)
 
 
-def test_decode_long_token_many_splits():
-    """A lone 8192-key decode on the TMA decode kernel: 128-key items give it
-    64 splits, two 32-split chunks in the merge kernel."""
+@pytest.mark.parametrize("split", [0, 128])
+def test_decode_long_token_many_splits(split):
+    """A lone 8192-key decode on the TMA decode kernel: 128-key items (chosen
+    by the planner for so few keys, or asked for) give it 64 splits, two
+    32-split chunks in the merge kernel."""
     sh = W.SHAPES["qwen"]
     ql, ctx, ph = [1, 1], [8192, 300], [1, 1]
     rng = np.random.default_rng(920)
     batch = W.build_batch(sh, ql, ctx, ph, rng, name="long_decode")
-    st = _step(batch)
+    st = _step(batch, split=split)
     assert st.plan.info()["decode_items"] >= 64
     out, lse = st.results()
     _compare(batch, out, lse)
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_decode_many_short_sequences(seed):
+    """300 decodes of 1..700 keys: more items than resident CTAs, so CTAs
+    take several items from the queue; also planned for 64 SMs."""
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(950 + seed)
+    ctx = rng.integers(1, 701, size=300).tolist()
+    batch = W.build_batch(sh, [1] * 300, ctx, [1] * 300, rng, name="short_decodes")
+    for sms in (0, 64):
+        st = _step(batch, sms=sms)
+        out, lse = st.results()
+        _compare(batch, out, lse)
 
 
 def test_decode_longest_context_split_cap():
