@@ -14,6 +14,7 @@ region.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the fp64 oracle on the host cores
   python bench.py --workload qwen_decode --kv-fp8   # decode over the FP8 (e4m3) cache
+  python bench.py --workload mla_prefill --mla-expand   # MLA prefill without absorption
 
 Under torchrun each rank runs an independent replica (seed + rank): the path
 has no exchange step, so there is no collective on the data path.
@@ -274,6 +275,157 @@ def run_reference(args):
     return 0
 
 
+def cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds: float = 15.0):
+    """Time the fp64 reference of the expanded MLA prefill: the latent append,
+    the expansion of every row (numpy), and the C oracle's attention on an
+    evenly spaced sample of the query rows, extrapolated by visible pairs."""
+    import oracle
+    from oracle import mla_expand as X
+    sh = batch.shape
+    t0 = time.perf_counter()
+    lat = oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping)
+    kb, vb = X.expand(lat, slots, ins["w_uk"], ins["w_uv"])
+    t_expand = time.perf_counter() - t0
+    kw = dict(num_q_heads=sh.num_q_heads, num_kv_heads=sh.num_q_heads, head_dim_qk=192, head_dim_v=128,
+              block_size=16)
+    target = max(1, W.pairs(batch) // 4096)
+    while True:
+        rows, sp, total = _sample_rows(batch, target_pairs=target)
+        t0 = time.perf_counter()
+        oracle.attention(batch.query_len, batch.context_len, bt, ins["q"], kb, vb, tokens=rows, **kw)
+        dt = time.perf_counter() - t0
+        if dt >= 0.2 or sp >= total:
+            break
+        target *= 4
+    rate = sp / max(dt, 1e-6)
+    rows, sp, total = _sample_rows(batch, target_pairs=int(rate * max(target_seconds - t_expand, 1.0)))
+    t0 = time.perf_counter()
+    oracle.attention(batch.query_len, batch.context_len, bt, ins["q"], kb, vb, tokens=rows, **kw)
+    t_sample = time.perf_counter() - t0
+    t_step = t_expand + t_sample * total / sp
+    return {"value": batch.num_tokens / t_step, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": (f"append + expansion of all {len(slots)} rows (numpy fp64), attention of {len(rows)} of "
+                       f"{batch.num_tokens} query rows ({sp / total:.4f} of the pairs, fp64 C oracle with OpenMP), "
+                       f"extrapolated by pairs"),
+            "sample_seconds": t_sample, "step_seconds_extrapolated": t_step}
+
+
+def run_fnpu_mla_expand(args):
+    """MLA prefill without absorption (latent append + expansion + MHA)."""
+    import torch
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import ExpandedMlaPrefill
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    fnpu.load()
+    peaks = _peaks()
+    batch = W.make_batch(args.workload, seed=args.seed + rank)
+    if not batch.shape.latent or np.any(batch.phase != 0):
+        raise SystemExit("--mla-expand needs a latent prefill workload (mla_prefill)")
+    ins = W.mla_expand_inputs(batch, seed=args.seed + rank)
+    slots, bt, nb = W.expanded_layout(batch)
+    st = ExpandedMlaPrefill(batch, ins["w_uk"], ins["w_uv"], ins["q"], slots, bt, nb, device=str(dev))
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_r = torch.zeros(L2_FLUSH_BYTES // 8, dtype=torch.float32, device=dev)
+    for _ in range(args.warmup):
+        _flush_l2(flush, flush_r)
+        st.run()
+    torch.cuda.synchronize(dev)
+    if fnpu.plan_check(st.plan) != fnpu.FNPU_OK or fnpu.check() != fnpu.FNPU_OK:
+        raise RuntimeError("device error flag raised during warm-up")
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clocks:
+        for i in range(K):
+            _flush_l2(flush, flush_r)
+            ev[i][0].record(stream)
+            st.append()
+            ev[i][1].record(stream)
+            st.expand()
+            ev[i][2].record(stream)
+            st.attend()
+            ev[i][3].record(stream)
+        torch.cuda.synchronize(dev)
+        if ws > 1:
+            torch.distributed.barrier()
+    clk = clocks.summary()
+    seg = [[ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(K)] for j in range(3)]
+    step_ms = max_over_ranks(sum(sum(x) for x in seg) / K, ws, dev)
+    t_app, t_exp, t_att = (sum(x) / K for x in seg)
+
+    bf = torch.bfloat16
+    h_q = torch.from_numpy(ins["q"]).view(bf).pin_memory()
+    h_k = torch.from_numpy(batch.k_new).view(bf).pin_memory()
+    h_s = torch.from_numpy(batch.slot_mapping).pin_memory()
+    h_o = torch.empty(st.out.shape, dtype=bf).pin_memory()
+    h_l = torch.empty(st.lse.shape, dtype=torch.float32).pin_memory()
+    h2d = sum(x.numel() * x.element_size() for x in (h_q, h_k, h_s))
+    d2h = h_o.numel() * h_o.element_size() + h_l.numel() * h_l.element_size()
+    e2e_ms = []
+    for i in range(args.warmup + K):
+        _flush_l2(flush, flush_r)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        st.q.copy_(h_q, non_blocking=True)
+        st.k_new.copy_(h_k, non_blocking=True)
+        st.slot_mapping.copy_(h_s, non_blocking=True)
+        st.run()
+        h_o.copy_(st.out, non_blocking=True)
+        h_l.copy_(st.lse, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        if i >= args.warmup:
+            e2e_ms.append(a.elapsed_time(b))
+    e2e = max_over_ranks(sum(e2e_ms) / len(e2e_ms), ws, dev)
+
+    H = batch.shape.num_q_heads
+    n = len(slots)
+    F_gemm = 2.0 * n * 512 * 128 * H * 2
+    F_attn = 2.0 * H * W.pairs(batch) * (192 + 128)
+    roof = {"bound": "tensor", "achieved": F_attn / (t_att * 1e-3) / 1e12, "peak": peaks["bf16_tflops"],
+            "unit": "TFLOP/s", "kernel": "prefill_mma_kernel<192, 128> (the attention call)"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = args.traffic
+    roof["peak_source"] = peaks["source"] + " burst"
+    T = batch.num_tokens
+    line = {
+        "metric": METRIC, "value": job_throughput(ws, T, step_ms), "unit": UNIT, "n_gpus": ws, "steps": K,
+        "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T, "path": "mla_expand",
+                   "expanded_rows": n, "heads": H, "flops_expand": F_gemm, "flops_attention": F_attn,
+                   "l2": "flushed between timed steps (512 MB write, then 256 MB read)", "plan": st.plan.info()},
+        "roofline": roof,
+        "roofline_step_frac": {"burst": (F_gemm + F_attn) / (peaks["bf16_tflops"] * 1e12) / (step_ms * 1e-3),
+                               "denominator": "(F_expand + F_attention) / bf16 peak of measured"},
+        "kernel_ms": {"append": t_app, "expand": t_exp, "attention": t_att},
+        "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
+        "gpu_launches": K * 3,  # append, gather, attention (plus two cuBLAS GEMM launches per step)
+        "clocks": clk,
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds=args.ref_seconds)
+    elif rank == 0:
+        line["cpu_baseline"] = None
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    return 0
+
+
 def _fp8_workload_ok(batch):
     if not np.all((batch.query_len == 1) & (batch.phase == 1)):
         raise SystemExit("--kv-fp8 needs a decode-only workload (qwen_decode)")
@@ -457,12 +609,17 @@ def main(argv=None):
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per attention launch, if measured for this kernel")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mla-expand", action="store_true",
+                    help="MLA prefill without absorption: latent rows expanded into per-head K/V, then MHA "
+                         "(latent prefill workloads: mla_prefill)")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="FP8 (e4m3) KV cache; decode-only workloads (qwen_decode)")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)  # at least three untimed warm-up steps
     if args.impl == "reference":
         return run_reference(args)
+    if args.mla_expand:
+        return run_fnpu_mla_expand(args)
     return run_fnpu(args)
 
 

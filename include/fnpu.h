@@ -278,6 +278,38 @@ const char *fnpu_last_cuda_error(void);
 /* Library version, major * 10000 + minor * 100 + patch. */
 int fnpu_version(void);
 
+/*
+ * MLA without absorption (prefill): expand latent cache rows into per-head
+ * keys and values, so that a prefill chunk can run as ordinary multi-head
+ * attention (d_qk = 192, d_v = 128, Hkv = Hq) through fnpu_mixed_attn_plan /
+ * _run over k_out / v_out seen as a paged cache. For row i with latent row
+ * L = latent_cache[slots[i]] (c = L[0:512], r = L[512:576]) and head h:
+ *   k_out[i, h, 0:128]   = c W_UK[h]      k_out[i, h, 128:192] = r
+ *   v_out[i, h, :]       = c W_UV[h]
+ * products in fp32, rounded to bf16 (nearest-even). This is the decompressed
+ * form of the latent attention of Sec. 4.1's DeepSeek-R1 deployment: with
+ * q = [q_nope, q_rope], q_nope . (c W_UK[h]) = (W_UK[h] q_nope) . c, so both
+ * forms give the same scores; the absorbed kernel of fnpu_mixed_attn_run
+ * attends over the latent rows directly.
+ *   desc          the latent cache: v_in_k_latent = 1, Hkv = 1, d_qk = 576,
+ *                 d_v = 512, block_size, num_blocks; num_q_heads = heads to expand
+ *   latent_cache  device bf16 [num_blocks, block_size, 576]
+ *   slots         device int64 [n]: latent slot of row i; negative = a zero row
+ *   w_uk, w_uv    device bf16 [Hq, 512, 128] (row-major per head)
+ *   workspace     device, at least n * 512 * 2 bytes (scratch; caller-owned)
+ *   k_out         device bf16 [n, Hq, 192];  v_out device bf16 [n, Hq, 128]
+ * The two products are cuBLAS strided-batched GEMMs on the stream (one
+ * batch entry per head); the gather is this library's kernel.
+ * Errors: FNPU_EINVAL for NULL or misaligned pointers (16 bytes; slots 8),
+ * n < 0 or a desc that is not a latent cache; FNPU_EUNSUPPORTED for other
+ * latent widths; FNPU_ECUDA if a CUDA or cuBLAS call fails. A slot >=
+ * num_blocks * block_size gives a zero row and raises the device error
+ * flag (FNPU_EDEVICE_RANGE from fnpu_check).
+ */
+int fnpu_mla_expand(const fnpu_attn_desc *desc, const void *latent_cache, const int64_t *slots, int32_t n,
+                    const void *w_uk, const void *w_uv, void *workspace, void *k_out, void *v_out,
+                    void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -40,7 +40,7 @@ EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
     "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error", "fnpu_plan_phase_ms",
-    "fnpu_dispatch_next_share",
+    "fnpu_dispatch_next_share", "fnpu_mla_expand",
 )
 
 
@@ -90,6 +90,7 @@ def load(build_if_missing: bool = True):
     lib.fnpu_mixed_attn_plan_ex.argtypes = [ctypes.POINTER(AttnDesc), i32, P, P, P, P, i32,
                                             ctypes.POINTER(PlanOpts), P, ctypes.POINTER(P)]
     lib.fnpu_mixed_attn_run.argtypes = [P, P, P, P, P, P, P]
+    lib.fnpu_mla_expand.argtypes = [ctypes.POINTER(AttnDesc), P, P, i32, P, P, P, P, P, P]
     lib.fnpu_plan_check.argtypes = [P, P]
     lib.fnpu_check.argtypes = [P]
     lib.fnpu_plan_destroy.argtypes = [P]
@@ -108,7 +109,7 @@ def load(build_if_missing: bool = True):
     for name in ("fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex",
                  "fnpu_mixed_attn_run", "fnpu_plan_check", "fnpu_check", "fnpu_plan_info",
                  "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_plan_phase_ms",
-                 "fnpu_dispatch_next_share"):
+                 "fnpu_dispatch_next_share", "fnpu_mla_expand"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -153,6 +154,18 @@ def _np(a, dtype) -> np.ndarray:
 # bytes of one block of the FP8 cache format (16 slots, 4 kv heads, d = 128):
 # K or V codes [16 * 4 * 128] then fp32 scales [16 * 4]
 FP8_BLOCK_BYTES = 16 * 4 * 128 + 16 * 4 * 4
+
+
+def mla_expand(desc: AttnDesc, latent_cache, slots, w_uk, w_uv, workspace, k_out, v_out, stream=None,
+               num_rows: Optional[int] = None) -> None:
+    """Per-head keys [n, Hq, 192] and values [n, Hq, 128] of latent rows
+    (``fnpu_mla_expand``): MLA prefill without absorption."""
+    if num_rows is None:
+        num_rows = int(slots.shape[0])
+    rc = load().fnpu_mla_expand(ctypes.byref(desc), _dptr(latent_cache), _dptr(slots), int(num_rows), _dptr(w_uk),
+                                _dptr(w_uv), _dptr(workspace), _dptr(k_out), _dptr(v_out), _stream(stream))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_mla_expand")
 
 
 def make_desc(num_q_heads, num_kv_heads, head_dim_qk, head_dim_v, block_size, num_blocks,

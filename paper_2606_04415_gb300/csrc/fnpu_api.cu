@@ -260,9 +260,12 @@ bool fp8_shape(const fnpu_attn_desc *d) {
 
 // Kernels exist for split K/V with d in {64, 128} (decode needs G <= 8) and
 // for the latent layout with d_qk = 576, d_v = 512 and a multiple of 64 heads.
-// The FP8 cache has a decode kernel only.
+// The FP8 cache has a decode kernel only; the per-head keys (192 columns) and
+// values (128) of a decompressed latent cache have a prefill kernel only.
 int kernel_support(const fnpu_attn_desc *d, bool has_decode, bool has_prefill) {
     if (d->kv_fp8) return fp8_shape(d) && !has_prefill ? FNPU_OK : FNPU_EUNSUPPORTED;
+    if (!d->v_in_k_latent && d->head_dim_qk == 192 && d->head_dim_v == 128)
+        return has_decode ? FNPU_EUNSUPPORTED : FNPU_OK;
     if (d->v_in_k_latent)
         return mla_supported(d->head_dim_qk, d->head_dim_v, d->num_q_heads, d->num_kv_heads) ? FNPU_OK
                                                                                                : FNPU_EUNSUPPORTED;

@@ -116,6 +116,10 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
                      const int64_t *slots, int32_t num_tokens, void *k_cache, void *v_cache,
                      void *stream);
 int read_and_clear_global_error(void *stream, int *flag);
+// MLA expansion: gather the c parts of latent rows (512 + 64 columns) into ws
+// [n, 512] and broadcast their r parts into columns 128..191 of k_out [n, heads, 192]
+int launch_mla_gather(const void *latent, const int64_t *slots, int32_t n, int64_t num_slots, int32_t heads,
+                      void *ws, void *k_out, void *stream);
 // FP8 (e4m3) cache: append (quantising) and decode (split-KV, TMA-fed)
 int launch_kv_append_fp8(const fnpu_attn_desc *d, const void *k_new, const void *v_new,
                          const int64_t *slots, int32_t num_tokens, void *k_cache, void *v_cache,

@@ -159,6 +159,52 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
     return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
 }
 
+// One warp per row: the 64 16-byte chunks of c into the workspace (two per
+// lane), then the 8 chunks of r into every head's key (lane e writes chunk
+// e mod 8 of heads e / 8, e / 8 + 4, ...). A negative slot gives a zero row;
+// a slot past the pool gives a zero row and raises the device error flag.
+// MLA expansion gather (latent rows of 512 + 64 columns; see mla_expand.cu).
+__global__ void __launch_bounds__(256) mla_gather_kernel(const uint4 *__restrict__ latent,
+                                                         const int64_t *__restrict__ slots, int32_t n,
+                                                         int64_t num_slots, int32_t heads,
+                                                         uint4 *__restrict__ ws, uint4 *__restrict__ k_out) {
+    const int lane = threadIdx.x & 31;
+    const int64_t step = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+    for (int64_t i = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5; i < n; i += step) {
+        int64_t s = __ldg(slots + i);
+        if (s >= num_slots) {
+            if (lane == 0) atomicOr(&g_device_error, 1);
+            s = -1;
+        }
+        const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+        const uint4 *row = latent + (s < 0 ? 0 : s) * (576 / 8);
+        uint4 *w = ws + i * (512 / 8);
+        w[lane] = s < 0 ? zero : __ldg(row + lane);
+        w[lane + 32] = s < 0 ? zero : __ldg(row + lane + 32);
+        const uint4 r = (lane < 64 / 8 && s >= 0) ? __ldg(row + 512 / 8 + lane) : zero;
+        uint4 rr;  // chunk lane mod 8 of r
+        rr.x = __shfl_sync(0xffffffffu, r.x, lane & 7);
+        rr.y = __shfl_sync(0xffffffffu, r.y, lane & 7);
+        rr.z = __shfl_sync(0xffffffffu, r.z, lane & 7);
+        rr.w = __shfl_sync(0xffffffffu, r.w, lane & 7);
+        uint4 *krow = k_out + i * heads * (192 / 8);
+        for (int e = lane; e < heads * (64 / 8); e += 32) krow[(e >> 3) * (192 / 8) + 128 / 8 + (e & 7)] = rr;
+    }
+}
+
+int launch_mla_gather(const void *latent, const int64_t *slots, int32_t n, int64_t num_slots, int32_t heads,
+                      void *ws, void *k_out, void *stream) {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (static_cast<int64_t>(n) + 7) / 8;  // 8 rows (warps) per block
+    const int grid = static_cast<int>(want < 16LL * sms ? want : 16LL * sms);
+    mla_gather_kernel<<<grid, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint4 *>(latent), slots, n, num_slots, heads, static_cast<uint4 *>(ws),
+        static_cast<uint4 *>(k_out));
+    return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
+}
+
 int read_and_clear_global_error(void *stream, int *flag) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(s) != cudaSuccess) return FNPU_ECUDA;

@@ -111,3 +111,73 @@ class DeviceStep:
         kc = self.k_cache.view(t.int16).cpu().numpy().view(np.uint16)
         vc = None if self.v_cache is None else self.v_cache.view(t.int16).cpu().numpy().view(np.uint16)
         return kc, vc
+
+
+class ExpandedMlaPrefill:
+    """MLA prefill without absorption, on device: the chunk's new latent rows
+    are appended (``fnpu_kv_append``), the latent rows of every sequence's
+    context are expanded (``fnpu_mla_expand``) into a paged cache of
+    per-head keys [n, Hq, 192] and values [n, Hq, 128] (each sequence from a
+    block boundary, blocks of 16), and the chunk runs as multi-head attention
+    over it through the ordinary plan / run.
+
+    ``batch``: a latent batch (its latent cache, block table and lengths; all
+    sequences are prefill chunks). ``slots``, ``block_table`` and
+    ``num_blocks`` give the expanded layout (host arrays, see
+    ``workloads.expanded_layout``); ``w_uk``, ``w_uv``, ``q`` are bf16 bits.
+    """
+
+    def __init__(self, batch, w_uk, w_uv, q, slots, block_table, num_blocks, device: str = "cuda",
+                 opts: Optional[PlanOpts] = None):
+        import torch
+        from . import mla_expand
+        self.torch = torch
+        self._expand = mla_expand
+        sh = batch.shape
+        H = sh.num_q_heads
+        bf = torch.bfloat16
+        self.latent_desc = make_desc(H, 1, sh.head_dim_qk, sh.head_dim_v, sh.block_size, batch.num_blocks, True)
+        self.desc = make_desc(H, H, 192, 128, 16, int(num_blocks))
+        self.latent = _to_dev(batch.k_cache, torch, bf, device)
+        self.k_new = _to_dev(batch.k_new, torch, bf, device)
+        self.slot_mapping = _to_dev(batch.slot_mapping, torch, None, device)
+        self.w_uk = _to_dev(w_uk, torch, bf, device)
+        self.w_uv = _to_dev(w_uv, torch, bf, device)
+        self.q = _to_dev(q, torch, bf, device)
+        self.slots = _to_dev(np.asarray(slots, np.int64), torch, None, device)
+        n = int(len(slots))
+        self.n = n
+        self.workspace = torch.empty((max(n, 1), 512), dtype=bf, device=device)
+        self.k = torch.empty((int(num_blocks) * 16, H, 192), dtype=bf, device=device)
+        self.v = torch.empty((int(num_blocks) * 16, H, 128), dtype=bf, device=device)
+        T = batch.num_tokens
+        self.out = torch.empty((T, H, 128), dtype=bf, device=device)
+        self.lse = torch.empty((T, H), dtype=torch.float32, device=device)
+        self.plan = mixed_attn_plan(self.desc, batch.query_len, batch.context_len, np.zeros(batch.num_seqs, np.uint8),
+                                    block_table, opts=opts)
+
+    def append(self, stream=None):
+        kv_append(self.latent_desc, self.k_new, None, self.slot_mapping, self.latent, None, stream=stream)
+
+    def expand(self, stream=None):
+        self._expand(self.latent_desc, self.latent, self.slots, self.w_uk, self.w_uv, self.workspace, self.k, self.v,
+                     stream=stream, num_rows=self.n)
+
+    def attend(self, stream=None):
+        mixed_attn_run(self.plan, self.q, self.k, self.v, self.out, self.lse, stream=stream)
+
+    def run(self, stream=None):
+        """One step: append the chunk's latent rows, expand, attention."""
+        self.append(stream)
+        self.expand(stream)
+        self.attend(stream)
+
+    def results(self):
+        self.torch.cuda.synchronize()
+        return (self.out.float().cpu().numpy(), self.lse.cpu().numpy())
+
+    def expanded_bits(self):
+        t = self.torch
+        t.cuda.synchronize()
+        return (self.k[:self.n].view(t.int16).cpu().numpy().view(np.uint16),
+                self.v[:self.n].view(t.int16).cpu().numpy().view(np.uint16))

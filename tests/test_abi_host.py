@@ -148,3 +148,24 @@ def test_fp8_cache_validation():
     rc = lib.fnpu_decode_attn_noalloc(ctypes.byref(fp8), 1, 16, 32, 4, 5, 0, 48, 64, 80, 96, 112, None)
     assert rc == fnpu.FNPU_EUNSUPPORTED
     assert fnpu.FP8_BLOCK_BYTES == 8448
+
+
+def test_mla_expand_validation_and_expanded_shape():
+    """fnpu_mla_expand rejects non-latent descriptors, other widths, bad
+    pointers; the expanded shape (192 / 128, Hkv = Hq) plans prefill only."""
+    lib = fnpu.load()
+    lat = fnpu.make_desc(128, 1, 576, 512, 64, 8, latent=True)
+    ok_ptrs = (16, 32, 4, 48, 64, 80, 96, 112)
+    assert lib.fnpu_mla_expand(ctypes.byref(lat), *ok_ptrs[:2], 0, *ok_ptrs[3:], None) == fnpu.FNPU_OK  # n = 0
+    assert lib.fnpu_mla_expand(ctypes.byref(lat), 16, 32, -1, 48, 64, 80, 96, 112, None) == fnpu.FNPU_EINVAL
+    assert lib.fnpu_mla_expand(ctypes.byref(lat), 16, 33, 4, 48, 64, 80, 96, 112, None) == fnpu.FNPU_EINVAL
+    assert lib.fnpu_mla_expand(ctypes.byref(lat), 16, 32, 4, 48, 64, 81, 96, 112, None) == fnpu.FNPU_EINVAL
+    assert lib.fnpu_mla_expand(ctypes.byref(lat), None, 32, 4, 48, 64, 80, 96, 112, None) == fnpu.FNPU_EINVAL
+    plain = fnpu.make_desc(**QWEN)
+    assert lib.fnpu_mla_expand(ctypes.byref(plain), 16, 32, 4, 48, 64, 80, 96, 112, None) == fnpu.FNPU_EINVAL
+    other = fnpu.make_desc(128, 1, 320, 256, 64, 8, latent=True)
+    assert lib.fnpu_mla_expand(ctypes.byref(other), 16, 32, 4, 48, 64, 80, 96, 112, None) == fnpu.FNPU_EUNSUPPORTED
+    exp = fnpu.make_desc(128, 128, 192, 128, 16, 100)
+    bt = np.zeros((1, 4), np.int32)
+    assert _plan_rc(exp, [1], [5], [1], bt) == fnpu.FNPU_EUNSUPPORTED   # no decode kernel for it
+    assert _plan_rc(exp, [3], [5], [0], bt) != fnpu.FNPU_EUNSUPPORTED   # prefill: valid (fails later without a GPU)

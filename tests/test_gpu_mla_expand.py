@@ -1,0 +1,97 @@
+"""MLA prefill without absorption on the GPU: latent rows expanded into
+per-head keys and values (fnpu_mla_expand: the library's gather kernel and two
+cuBLAS GEMMs), then multi-head attention (d_qk 192, d_v 128) over them through
+the plan / run, against the fp64 reference (oracle.mla_expand + the C oracle).
+
+Expanded rows: the rotary part is a copy (bit-exact); the products are fp32
+sums rounded to bf16 against the reference's exactly rounded fp64 sums, so an
+element may differ by one bf16 unit where the fp32 sum lands on the other side
+of a rounding boundary (rare). Attention: |O - O_ref| <= 2e-2, |LSE - LSE_ref|
+<= 1e-3, the reference run on its own expanded rows.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import workloads as W
+from oracle import mla_expand as X
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+O_TOL = 2e-2
+LSE_TOL = 1e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2606_04415_gb300 as fnpu
+    fnpu.load()
+
+
+def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import ExpandedMlaPrefill
+    rng = np.random.default_rng(seed)
+    sh = W.Shape(heads, 1, 576, 512, bs, True)
+    batch = W.build_batch(sh, q_lens, ctxs, [0] * len(q_lens), rng, name="mla_expand")
+    ins = W.mla_expand_inputs(batch, seed)
+    slots, bt, nb = W.expanded_layout(batch)
+    st = ExpandedMlaPrefill(batch, ins["w_uk"], ins["w_uv"], ins["q"], slots, bt, nb)
+    st.run()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK and fnpu.check() == fnpu.FNPU_OK
+    out, lse = st.results()
+    gk, gv = st.expanded_bits()
+    lat = oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping)
+    kb, vb = X.expand(lat, slots, ins["w_uk"], ins["w_uv"])
+    # rotary part copied, products within one bf16 unit and nearly all exact
+    assert np.array_equal(gk[:, :, 128:], kb[:, :, 128:])
+    for g, r in ((gk[:, :, :128], kb[:, :, :128]), (gv, vb)):
+        gf, rf = X.bf16_bits_to_f64(g), X.bf16_bits_to_f64(r)
+        assert np.all(np.abs(gf - rf) <= np.abs(rf) * 2.0 ** -7 + 1e-30)
+        assert np.mean(g == r) > 0.99
+    ref_o, ref_l = oracle.attention(batch.query_len, batch.context_len, bt, ins["q"], kb, vb, num_q_heads=heads,
+                                    num_kv_heads=heads, head_dim_qk=192, head_dim_v=128, block_size=16,
+                                    tokens=tokens)
+    if tokens is not None:
+        out, lse = out[tokens], lse[tokens]
+    assert np.isfinite(out).all() and np.isfinite(lse).all()
+    eo, el = np.abs(out - ref_o).max(), np.abs(lse - ref_l).max()
+    assert eo <= O_TOL, f"max |dO| = {eo}"
+    assert el <= LSE_TOL, f"max |dLSE| = {el}"
+    return st
+
+
+@pytest.mark.parametrize("heads", [128, 16])
+def test_ragged_chunks_on_prefixes(heads):
+    """Chunks of 1, 17, 64 and 200 rows on prefixes of 0, 23, 300 and 824
+    (rows and keys off every tile boundary), latent blocks of 64."""
+    _run([1, 17, 64, 200], [1, 40, 364, 1024], heads=heads, seed=1)
+
+
+def test_latent_blocks_of_16():
+    _run([33, 128], [33, 500], heads=128, seed=2, bs=16)
+
+
+def test_full_size_prefill_chunk_sampled_rows():
+    """The 1024-token DeepSeek-R1 prefill chunk of the MLA co-located workload
+    (no prefix, 128 heads): all of it expanded and attended on the GPU, the
+    reference on rows at tile boundaries and at random."""
+    rng = np.random.default_rng(5)
+    rows = sorted({0, 1, 63, 64, 127, 128, 511, 512, 1023} | set(rng.integers(0, 1024, 12).tolist()))
+    _run([1024], [1024], heads=128, seed=3, tokens=np.asarray(rows, np.int64))
+
+
+def test_out_of_range_slot_gives_zero_row_and_flag():
+    import paper_2606_04415_gb300 as fnpu
+    st = _run([8], [8], heads=16, seed=4)
+    bad = torch.tensor([st.latent_desc.num_blocks * st.latent_desc.block_size + 5, -1], dtype=torch.int64,
+                       device="cuda")
+    k = torch.full((2, 16, 192), 1.0, dtype=torch.bfloat16, device="cuda")
+    v = torch.full((2, 16, 128), 1.0, dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty((2, 512), dtype=torch.bfloat16, device="cuda")
+    fnpu.mla_expand(st.latent_desc, st.latent, bad, st.w_uk, st.w_uv, ws, k, v)
+    assert fnpu.check() == fnpu.FNPU_EDEVICE_RANGE
+    assert not k.float().abs().sum().item() and not v.float().abs().sum().item()

@@ -40,7 +40,7 @@ import numpy as np
 
 BF16_CANARY = np.uint16(0x7FC1)  # a quiet NaN with a distinct payload
 
-CONFIG_NAMES = ("tiny", "qwen_decode", "qwen_prefill", "qwen_coloc", "mla_coloc", "mla_coloc_small")
+CONFIG_NAMES = ("tiny", "qwen_decode", "qwen_prefill", "qwen_coloc", "mla_coloc", "mla_coloc_small", "mla_prefill")
 
 
 @dataclasses.dataclass(frozen=True)
@@ -164,6 +164,10 @@ def draw_lengths(name: str, rng: np.random.Generator):
         q = [256] + [1] * 48
         ctx = [256] + dec.tolist()
         ph = [0] + [1] * 48
+    elif name == "mla_prefill":
+        # the prefill chunk of the MLA co-located mix alone: one 1024-token
+        # prompt, no prefix (for the expanded, non-absorbed prefill path)
+        q, ctx, ph = [1024], [1024], [0]
     else:
         raise ValueError(f"unknown workload {name!r}")
     return (np.asarray(q, np.int32), np.asarray(ctx, np.int32), np.asarray(ph, np.uint8))
@@ -287,6 +291,45 @@ def stale_pool_bytes(nbytes: int, seed: int) -> tuple:
     kernel that reads a slot it must not see goes wrong visibly."""
     rng = np.random.default_rng([seed, 0xF8])
     return (rng.integers(0, 256, nbytes, dtype=np.uint8), rng.integers(0, 256, nbytes, dtype=np.uint8))
+
+
+def mla_expand_inputs(batch: Batch, seed: int = 0) -> dict:
+    """Inputs of MLA prefill without absorption on a latent batch: the per-head
+    up-projections W_UK, W_UV (bf16 [Hq, 512, 128], N(0, 1/512) so that the
+    expanded keys and values are about N(0, 1)) and the decompressed queries
+    [T, Hq, 192] (N(0, 1)), all seeded."""
+    sh = batch.shape
+    if not sh.latent:
+        raise ValueError("a latent batch is needed")
+    rng = np.random.default_rng([seed, 0x3A])
+    H = sh.num_q_heads
+    w_uk = f32_to_bf16_bits((rng.standard_normal((H, 512, 128)) / math.sqrt(512)).astype(np.float32))
+    w_uv = f32_to_bf16_bits((rng.standard_normal((H, 512, 128)) / math.sqrt(512)).astype(np.float32))
+    q = _normal_bf16(rng, (batch.num_tokens, H, 192))
+    return {"w_uk": w_uk, "w_uv": w_uv, "q": q}
+
+
+def expanded_layout(batch: Batch, block_size: int = 16) -> tuple:
+    """Rows of the expanded cache of a latent batch: every sequence's positions
+    0..ctx-1 in order, each sequence starting on a block boundary (padding rows
+    have slot -1). Returns (slots int64 [n], block_table int32 [S, width],
+    num_blocks): block_table[s][j] is the expanded block of position 16 j."""
+    bs_l = batch.shape.block_size
+    S = batch.num_seqs
+    nblk = [(int(c) + block_size - 1) // block_size for c in batch.context_len]
+    width = max(nblk) if nblk else 1
+    bt = np.zeros((S, width), np.int32)
+    slots = []
+    first = 0
+    for s in range(S):
+        c = int(batch.context_len[s])
+        pos = np.arange(c, dtype=np.int64)
+        sl = batch.block_table[s, pos // bs_l].astype(np.int64) * bs_l + pos % bs_l
+        pad = nblk[s] * block_size - c
+        slots.append(np.concatenate([sl, np.full(pad, -1, np.int64)]))
+        bt[s, :nblk[s]] = np.arange(first, first + nblk[s])
+        first += nblk[s]
+    return (np.concatenate(slots) if slots else np.zeros(0, np.int64)), bt, max(first, 1)
 
 
 def pairs(batch: Batch) -> int:
