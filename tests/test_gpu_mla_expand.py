@@ -6,8 +6,15 @@ the plan / run, against the fp64 reference (oracle.mla_expand + the C oracle).
 Expanded rows: the rotary part is a copy (bit-exact); the products are fp32
 sums rounded to bf16 against the reference's exactly rounded fp64 sums, so an
 element may differ by one bf16 unit where the fp32 sum lands on the other side
-of a rounding boundary (rare). Attention: |O - O_ref| <= 2e-2, |LSE - LSE_ref|
-<= 1e-3, the reference run on its own expanded rows.
+of a rounding boundary (about 1% of them, asserted below).
+
+Attention kernel alone (random 192-wide keys and 128-wide values from the
+seeded generator): |O - O_ref| <= 2e-2, |LSE - LSE_ref| <= 1e-3 as for every
+attention path. End to end (expansion then attention), the reference runs on
+its own expanded rows; a key element one bf16 unit off moves a score by up to
+scale * |q_d| * 2^-7 |k_d| (about 5e-4 for N(0, 1) data at the tails), and a
+few such elements in a row move the log-sum-exp by up to about 2e-3: the LSE
+bound there is 3e-3 (O stays 2e-2).
 """
 import numpy as np
 import pytest
@@ -21,6 +28,7 @@ pytestmark = pytest.mark.gpu
 
 O_TOL = 2e-2
 LSE_TOL = 1e-3
+LSE_TOL_EXPANDED = 3e-3  # end to end: flipped bf16 roundings of the expanded keys (see above)
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -46,11 +54,16 @@ def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
     gk, gv = st.expanded_bits()
     lat = oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping)
     kb, vb = X.expand(lat, slots, ins["w_uk"], ins["w_uv"])
-    # rotary part copied, products within one bf16 unit and nearly all exact
+    # rotary part copied; products within one bf16 unit plus the fp32
+    # accumulation error (512 terms: at most 2^-15 of the sum of |terms|,
+    # doubled), and nearly all bit-exact
     assert np.array_equal(gk[:, :, 128:], kb[:, :, 128:])
-    for g, r in ((gk[:, :, :128], kb[:, :, :128]), (gv, vb)):
+    c_abs = np.abs(X.latent_rows(lat, slots)[:, :512])
+    for g, r, w in ((gk[:, :, :128], kb[:, :, :128], ins["w_uk"]), (gv, vb, ins["w_uv"])):
         gf, rf = X.bf16_bits_to_f64(g), X.bf16_bits_to_f64(r)
-        assert np.all(np.abs(gf - rf) <= np.abs(rf) * 2.0 ** -7 + 1e-30)
+        s_abs = np.einsum("nk,hkd->nhd", c_abs, np.abs(X.bf16_bits_to_f64(w)))
+        bound = np.abs(rf) * 2.0 ** -7 + s_abs * 2.0 ** -14
+        assert np.all(np.abs(gf - rf) <= bound), float(np.max(np.abs(gf - rf) - bound))
         assert np.mean(g == r) > 0.99
     ref_o, ref_l = oracle.attention(batch.query_len, batch.context_len, bt, ins["q"], kb, vb, num_q_heads=heads,
                                     num_kv_heads=heads, head_dim_qk=192, head_dim_v=128, block_size=16,
@@ -60,8 +73,27 @@ def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
     assert np.isfinite(out).all() and np.isfinite(lse).all()
     eo, el = np.abs(out - ref_o).max(), np.abs(lse - ref_l).max()
     assert eo <= O_TOL, f"max |dO| = {eo}"
-    assert el <= LSE_TOL, f"max |dLSE| = {el}"
+    assert el <= LSE_TOL_EXPANDED, f"max |dLSE| = {el}"
     return st
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_attention_kernel_on_192_128_heads(seed):
+    """The mma.sync prefill kernel for 192-wide keys and 128-wide values, one
+    kv head per query head (the expanded MLA shape), on random bf16 caches:
+    ragged chunks on prefixes, all rows, the attention tolerances."""
+    from paper_2606_04415_gb300.step import DeviceStep
+    import paper_2606_04415_gb300 as fnpu
+    rng = np.random.default_rng(60 + seed)
+    sh = W.Shape(16, 16, 192, 128, 16, False)
+    batch = W.build_batch(sh, [1, 17, 64, 130], [1, 40, 364, 700], [0, 0, 0, 0], rng, name="mha192")
+    st = DeviceStep(batch)
+    st.run()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
+    out, lse = st.results()
+    ref_o, ref_l, _, _ = oracle.run_step(batch)
+    assert np.isfinite(out).all()
+    assert np.abs(out - ref_o).max() <= O_TOL and np.abs(lse - ref_l).max() <= LSE_TOL
 
 
 @pytest.mark.parametrize("heads", [128, 16])
