@@ -61,8 +61,9 @@ typedef enum {
 typedef struct {
     int32_t num_q_heads;   /* Hq, a multiple of num_kv_heads */
     int32_t num_kv_heads;  /* Hkv (1 for the latent layout) */
-    int32_t head_dim_qk;   /* supported: 64, 128 (split K/V); 576 (latent) */
-    int32_t head_dim_v;    /* = head_dim_qk for split K/V; 512 for latent */
+    int32_t head_dim_qk;   /* supported: 64, 128 (split K/V); 576 (latent); 192 (expanded
+                              latent rows, see fnpu_mla_expand: prefill plans only) */
+    int32_t head_dim_v;    /* = head_dim_qk for split K/V; 512 for latent; 128 with 192 */
     int32_t block_size;    /* tokens per KV block (16 or 64 ...), >= 1 */
     int32_t num_blocks;    /* blocks in the pool */
     int32_t v_in_k_latent; /* 1: MLA latent cache, V aliases K[:, :d_v] */
