@@ -208,3 +208,42 @@ def decode_attention(context_len, block_table, q_bf16, k_pool, v_pool, *, num_q_
             out[s, h] = (w[:, None] * vals[:, kvh, :]).sum(0) / l
             lse[s, h] = m + np.log(l)
     return out, lse
+
+
+def attention(query_len, context_len, block_table, q_bf16, k_pool, v_pool, *, num_q_heads: int, num_kv_heads: int,
+              scale: float = 0.0, tokens=None) -> tuple:
+    """Output (float64 [rows, Hq, d]) and LSE (float64 [rows, Hq]) of a mixed
+    step over the dequantised cache: sequence s's query i sits at position
+    ctx_s - q_s + i and attends causally to keys 0..pos (keys of sequence s
+    at block_table[s][j / 16], offset j % 16); softmax(q k^T * scale) v with
+    k, v = code value * row scale. Queries are packed sequence by sequence;
+    `tokens` selects output rows (default all)."""
+    k_codes, k_scales, v_codes, v_scales = unpack_pools(k_pool, v_pool, num_kv_heads)
+    g = num_q_heads // num_kv_heads
+    sc = scale if scale > 0 else 1.0 / np.sqrt(D)
+    qf = bf16_bits_to_f32(q_bf16).astype(np.float64).reshape(-1, num_q_heads, D)
+    ql = np.asarray(query_len, np.int64)
+    cl = np.asarray(context_len, np.int64)
+    starts = np.concatenate([[0], np.cumsum(ql)])
+    T = int(starts[-1])
+    rows = np.arange(T) if tokens is None else np.asarray(tokens, np.int64)
+    out = np.zeros((rows.size, num_q_heads, D))
+    lse = np.zeros((rows.size, num_q_heads))
+    seq_of = np.searchsorted(starts, rows, side="right") - 1
+    for s in np.unique(seq_of):
+        c = int(cl[s])
+        idx = np.arange(c)
+        blk = np.asarray(block_table)[s, idx // BS]
+        keys = e4m3_decode(k_codes[blk, idx % BS]) * k_scales[blk, idx % BS][..., None].astype(np.float64)
+        vals = e4m3_decode(v_codes[blk, idx % BS]) * v_scales[blk, idx % BS][..., None].astype(np.float64)
+        for ri in np.flatnonzero(seq_of == s):
+            t = int(rows[ri])
+            pos = c - int(ql[s]) + (t - int(starts[s]))
+            for h in range(num_q_heads):
+                kvh = h // g
+                x = keys[:pos + 1, kvh, :] @ qf[t, h] * sc
+                m = x.max()
+                w = np.exp(x - m)
+                out[ri, h] = (w[:, None] * vals[:pos + 1, kvh, :]).sum(0) / w.sum()
+                lse[ri, h] = m + np.log(w.sum())
+    return out, lse

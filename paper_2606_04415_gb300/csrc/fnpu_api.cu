@@ -260,10 +260,12 @@ bool fp8_shape(const fnpu_attn_desc *d) {
 
 // Kernels exist for split K/V with d in {64, 128} (decode needs G <= 8) and
 // for the latent layout with d_qk = 576, d_v = 512 and a multiple of 64 heads.
-// The FP8 cache has a decode kernel only; the per-head keys (192 columns) and
-// values (128) of a decompressed latent cache have a prefill kernel only.
+// The FP8 cache has one decode and one prefill kernel for its one shape; the
+// per-head keys (192 columns) and values (128) of a decompressed latent cache
+// have a prefill kernel only.
 int kernel_support(const fnpu_attn_desc *d, bool has_decode, bool has_prefill) {
-    if (d->kv_fp8) return fp8_shape(d) && !has_prefill ? FNPU_OK : FNPU_EUNSUPPORTED;
+    (void)has_prefill;
+    if (d->kv_fp8) return fp8_shape(d) ? FNPU_OK : FNPU_EUNSUPPORTED;
     if (!d->v_in_k_latent && d->head_dim_qk == 192 && d->head_dim_v == 128)
         return has_decode ? FNPU_EUNSUPPORTED : FNPU_OK;
     if (d->v_in_k_latent)
@@ -399,7 +401,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                      mla_tc_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_q_heads, desc->num_kv_heads, bs);
     pl->use_dt = !pl->use_mla && decode_tma_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_kv_heads,
                                                       desc->num_q_heads / desc->num_kv_heads, bs);
-    pl->use_tc = !pl->use_mla && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
+    pl->use_tc = !pl->use_mla && !desc->kv_fp8 && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
                  prefill_tc_supported(desc->head_dim_qk, desc->head_dim_v, bs,
                                       desc->num_q_heads / desc->num_kv_heads);
 
@@ -821,6 +823,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
              : pl->use_dt    ? launch_decode_tma(p, stream, 3 * pl->num_sms)
                              : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
+    if (pl->desc.kv_fp8) return launch_prefill_fp8(p, stream);
     return pl->use_tc ? launch_prefill_tc(p, stream, pl->num_sms) : launch_prefill_mma(p, stream);
 }
 

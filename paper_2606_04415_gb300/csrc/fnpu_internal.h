@@ -125,6 +125,7 @@ int launch_kv_append_fp8(const fnpu_attn_desc *d, const void *k_new, const void 
                          const int64_t *slots, int32_t num_tokens, void *k_cache, void *v_cache,
                          void *stream);
 int launch_decode_fp8(const AttnParams &p, void *stream, int max_ctas);
+int launch_prefill_fp8(const AttnParams &p, void *stream);
 bool decode_fp8_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_decode_mma(const AttnParams &p, void *stream);
 int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas);

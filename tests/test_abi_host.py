@@ -125,9 +125,9 @@ def test_append_and_run_reject_null_pointers():
 
 
 def test_fp8_cache_validation():
-    """The FP8 cache: kv_fp8 outside {0, 1} is invalid; other shapes, latent
-    caches and plans with prefill work are unsupported; all decided on the
-    host before any CUDA call."""
+    """The FP8 cache: kv_fp8 outside {0, 1} is invalid; other shapes and latent
+    caches are unsupported; all decided on the host before any CUDA call.
+    Plans with prefill work are valid (without a GPU they fail later)."""
     lib = fnpu.load()
     bt = np.zeros((2, 4), np.int32)
     bad = fnpu.make_desc(**QWEN)
@@ -135,8 +135,8 @@ def test_fp8_cache_validation():
     assert _plan_rc(bad, [1], [5], [1], bt[:1]) == fnpu.FNPU_EINVAL
     assert lib.fnpu_kv_append(ctypes.byref(bad), 16, 32, 64, 4, 128, 256, None) == fnpu.FNPU_EINVAL
     fp8 = fnpu.make_desc(**QWEN, kv_fp8=True)
-    assert _plan_rc(fp8, [8, 1], [8, 20], [0, 1], bt) == fnpu.FNPU_EUNSUPPORTED      # prefill chunk
-    assert _plan_rc(fp8, [3], [20], [1], bt[:1]) == fnpu.FNPU_EUNSUPPORTED          # multi-token decode
+    assert _plan_rc(fp8, [8, 1], [8, 20], [0, 1], bt) not in (fnpu.FNPU_EUNSUPPORTED, fnpu.FNPU_EINVAL)
+    assert _plan_rc(fp8, [3], [20], [1], bt[:1]) not in (fnpu.FNPU_EUNSUPPORTED, fnpu.FNPU_EINVAL)
     for other in (dict(head_dim_qk=64, head_dim_v=64), dict(num_kv_heads=2, num_q_heads=14),
                   dict(block_size=32), dict(num_q_heads=36)):
         d = fnpu.make_desc(**dict(QWEN, **other), kv_fp8=True)

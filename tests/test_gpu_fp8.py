@@ -30,12 +30,13 @@ def _cuda():
     fnpu.load()
 
 
-def _batch(ctx, hq=28, seed=0, slack=1.25):
+def _batch(ctx, hq=28, seed=0, slack=1.25, ql=None, phase=None):
     rng = np.random.default_rng(seed)
     S = len(ctx)
     shape = W.Shape(hq, 4, 128, 128, 16, False)
-    return W.build_batch(shape, np.ones(S, np.int32), np.asarray(ctx, np.int32), np.ones(S, np.uint8), rng,
-                         name="fp8", seed=seed, pool_slack=slack)
+    ql = np.ones(S, np.int32) if ql is None else np.asarray(ql, np.int32)
+    phase = np.ones(S, np.uint8) if phase is None else np.asarray(phase, np.uint8)
+    return W.build_batch(shape, ql, np.asarray(ctx, np.int32), phase, rng, name="fp8", seed=seed, pool_slack=slack)
 
 
 def _reference_pools(batch, init, seqs=None):
@@ -72,9 +73,15 @@ def _run(batch, seed=0, split=0, check_pools=True):
     return st, out, lse, kp, vp
 
 
-def _compare(batch, out, lse, kp, vp):
-    ref_o, ref_l = F8.decode_attention(batch.context_len, batch.block_table, batch.q, kp, vp,
-                                       num_q_heads=batch.shape.num_q_heads, num_kv_heads=4)
+def _compare(batch, out, lse, kp, vp, tokens=None):
+    if np.all(batch.query_len == 1) and tokens is None:
+        ref_o, ref_l = F8.decode_attention(batch.context_len, batch.block_table, batch.q, kp, vp,
+                                           num_q_heads=batch.shape.num_q_heads, num_kv_heads=4)
+    else:
+        ref_o, ref_l = F8.attention(batch.query_len, batch.context_len, batch.block_table, batch.q, kp, vp,
+                                    num_q_heads=batch.shape.num_q_heads, num_kv_heads=4, tokens=tokens)
+        if tokens is not None:
+            out, lse = out[tokens], lse[tokens]
     assert np.isfinite(out).all() and np.isfinite(lse).all()
     eo, el = np.abs(out - ref_o).max(), np.abs(lse - ref_l).max()
     assert eo <= O_TOL, f"max |dO| = {eo}"
@@ -172,3 +179,36 @@ def test_fp8_plan_reuse_runs_repeatedly():
     o2, l2 = st.results()
     assert np.array_equal(out, o2) and np.array_equal(lse, l2)
     _compare(batch, o2, l2, kp, vp)
+
+
+@pytest.mark.parametrize("hq", [28, 32])
+def test_fp8_mixed_step_prefill_and_decode(hq):
+    """Prefill chunks on prefixes (64 rows on none, 130 on 170), a 3-token
+    decode (the prefill queue) and one-token decodes (one of 2049 keys) over
+    the FP8 cache: the prefill rows run on the f16 mma.sync FP8 prefill kernel,
+    the decodes on the FP8 decode kernel; all rows against the reference."""
+    batch = _batch([64, 500, 300, 200, 2049], hq=hq, seed=7, ql=[64, 1, 130, 3, 1], phase=[0, 1, 0, 1, 1])
+    _, out, lse, kp, vp = _run(batch, seed=7)
+    _compare(batch, out, lse, kp, vp)
+
+
+def test_fp8_colocated_workload_sampled_rows():
+    """The co-located Qwen workload over the FP8 cache (one 2048-token chunk on
+    a prefix of 6969 + 128 decodes, seed 0) at full size; the reference fills
+    the blocks of the chunk's sequence and of 6 decodes and recomputes rows at
+    tile boundaries of the chunk, random rows and those decodes."""
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    batch = W.make_batch("qwen_coloc", seed=0)
+    init = W.stale_pool_bytes(batch.num_blocks * F8.block_bytes(4), 0)
+    st = DeviceStep(batch, kv_fp8=True, pool_init=init)
+    st.run()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK and fnpu.check() == fnpu.FNPU_OK
+    out, lse = st.results()
+    rng = np.random.default_rng(12)
+    dec = sorted(rng.choice(np.arange(1, batch.num_seqs), 6, replace=False).tolist())
+    seqs = [0] + dec
+    kp, vp = _reference_pools(batch, init, seqs)
+    rows = sorted({0, 1, 63, 64, 65, 127, 1023, 1024, 2047} | set(rng.integers(0, 2048, 10).tolist()))
+    tokens = np.asarray(rows + [int(batch.query_start[s]) for s in dec], np.int64)
+    _compare(batch, out, lse, kp, vp, tokens=tokens)

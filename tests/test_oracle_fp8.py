@@ -152,3 +152,32 @@ def test_binade_rounding_equals_the_table_search():
     near = np.concatenate([np.nextafter(mids, np.float32(0)), np.nextafter(mids, np.float32(1e9))])
     for arr in (x, vals.astype(np.float32), mids, -mids, near, np.array([0, -0.0, 448, 449, 470, 1e38], np.float32)):
         assert np.array_equal(fp8.e4m3_round(arr), fp8.e4m3_round_by_search(arr))
+
+
+def test_mixed_step_matches_the_bf16_oracle_when_every_scale_is_one():
+    """Prefill chunks on prefixes, a multi-token decode and decodes: with every
+    scale 1 the fp8 reference equals the bf16 C oracle on the dequantised cache
+    (causal rows at absolute positions, sampled and whole)."""
+    rng = np.random.default_rng(8)
+    hkv, hq, nb = 4, 28, 12
+    vals = np.array([fp8.e4m3_value(c) for c in range(127)], np.float32)
+    def rows(n):
+        x = rng.choice(np.concatenate([vals, -vals[1:]]), size=(n, 16, hkv, 128)).astype(np.float32) / 64
+        x[..., 0] = 448.0
+        return x
+    kc, ks = fp8.quantize_rows(_bf16(rows(nb)))
+    vc, vs = fp8.quantize_rows(_bf16(rows(nb)))
+    kp, vp = fp8.pack_pools(kc, ks, vc, vs)
+    ql = np.array([20, 1, 3, 1], np.int32)
+    cl = np.array([50, 77, 40, 1], np.int32)
+    bt = rng.integers(0, nb, size=(4, 5)).astype(np.int32)  # blocks may repeat: both sides read the same
+    q = _bf16(rng.standard_normal((int(ql.sum()), hq, 128)))
+    kdq = _bf16(fp8.e4m3_decode(kc).astype(np.float32))
+    vdq = _bf16(fp8.e4m3_decode(vc).astype(np.float32))
+    ref_o, ref_l = oracle.attention(ql, cl, bt, q, kdq, vdq, num_q_heads=hq, num_kv_heads=hkv, head_dim_qk=128,
+                                    head_dim_v=128, block_size=16)
+    out, lse = fp8.attention(ql, cl, bt, q, kp, vp, num_q_heads=hq, num_kv_heads=hkv)
+    assert np.abs(out - ref_o).max() < 1e-12 and np.abs(lse - ref_l).max() < 1e-12
+    tok = np.array([0, 19, 21, 23, 24])
+    o2, l2 = fp8.attention(ql, cl, bt, q, kp, vp, num_q_heads=hq, num_kv_heads=hkv, tokens=tok)
+    assert np.array_equal(o2, out[tok]) and np.array_equal(l2, lse[tok])
