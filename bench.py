@@ -216,63 +216,52 @@ def cpu_baseline(batch, target_seconds: float = 15.0, reps: int = 1):
 
 def cpu_baseline_fp8(batch, target_seconds: float = 15.0):
     """Time the fp64 FP8 reference: the step's append (all new rows, on the
-    whole pool) and the decode attention of an evenly spaced sample of the
-    sequences, extrapolated to all of them by keys. The sampled sequences'
-    prefix rows are put into the reference pools first, untimed."""
+    whole pool) and the attention of an evenly spaced sample of the query rows,
+    extrapolated to the step by visible pairs. The sampled rows' sequences get
+    their prefix rows into the reference pools first, untimed."""
     from oracle import fp8 as F8
     sh = batch.shape
     init = W.stale_pool_bytes(batch.num_blocks * F8.block_bytes(sh.num_kv_heads), batch.seed)
-    ctx = batch.context_len.astype(np.int64)
-    # the reference decodes about 25k keys a second (d = 128, 28 heads) and
-    # fills its pools about 8 times slower: a tenth of the budget for the
-    # decode sample keeps the whole call near the budget; at least one sequence
-    want = max(1, min(batch.num_seqs, int(round(batch.num_seqs * min(1.0, 25000 * target_seconds / 10 / ctx.sum())))))
-    seqs = np.unique(np.linspace(0, batch.num_seqs - 1, want).round().astype(np.int64))
-    k, v, sl = W.prefix_rows(batch)
-    pre = ctx - batch.query_len
-    p0 = np.concatenate([[0], np.cumsum(pre)])
-    pi = np.concatenate([np.arange(p0[s], p0[s + 1]) for s in seqs])
-    kp, vp = F8.kv_append(init[0], init[1], k[pi], v[pi], sl[pi], sh.num_kv_heads)
+    starts = batch.query_start
+    seq_q = np.repeat(np.arange(batch.num_seqs), batch.query_len)
+    pos = batch.context_len[seq_q] - batch.query_len[seq_q] + (np.arange(batch.num_tokens) - starts[seq_q])
+    row_pairs = (pos + 1).astype(np.int64)
+
+    def pick(n):
+        return np.unique(np.linspace(0, batch.num_tokens - 1, min(n, batch.num_tokens)).round().astype(np.int64))
+
+    def pools_for(rows):  # the reference pools with the prefix rows of the rows' sequences
+        seqs = np.unique(seq_q[rows])
+        k, v, sl = W.prefix_rows(batch)
+        pre = (batch.context_len - batch.query_len).astype(np.int64)
+        p0 = np.concatenate([[0], np.cumsum(pre)])
+        pi = np.concatenate([np.arange(p0[s], p0[s + 1]) for s in seqs])
+        return F8.kv_append(init[0], init[1], k[pi], v[pi], sl[pi], sh.num_kv_heads)
+
+    # calibrate on 4 rows, then take about a third of the budget of rows
+    rows = pick(4)
+    kp, vp = pools_for(rows)  # (the step's own rows are not in yet: the time does not depend on values)
+    t0 = time.perf_counter()
+    F8.attention(batch.query_len, batch.context_len, batch.block_table, batch.q, kp, vp,
+                 num_q_heads=sh.num_q_heads, num_kv_heads=sh.num_kv_heads, tokens=rows)
+    per_pair = (time.perf_counter() - t0) / float(row_pairs[rows].sum())
+    n = int(target_seconds / 3 / max(per_pair * float(row_pairs.mean()), 1e-9))
+    rows = pick(max(4, n))
+    kp, vp = pools_for(rows)
     t0 = time.perf_counter()
     kp, vp = F8.kv_append(kp, vp, batch.k_new, batch.v_new, batch.slot_mapping, sh.num_kv_heads)
     t_append = time.perf_counter() - t0
     t0 = time.perf_counter()
-    F8.decode_attention(ctx[seqs], batch.block_table[seqs], batch.q[batch.query_start[seqs]], kp, vp,
-                        num_q_heads=sh.num_q_heads, num_kv_heads=sh.num_kv_heads)
+    F8.attention(batch.query_len, batch.context_len, batch.block_table, batch.q, kp, vp,
+                 num_q_heads=sh.num_q_heads, num_kv_heads=sh.num_kv_heads, tokens=rows)
     t_sample = time.perf_counter() - t0
-    frac = float(ctx[seqs].sum()) / float(ctx.sum())
+    frac = float(row_pairs[rows].sum()) / float(row_pairs.sum())
     t_step = t_append + t_sample / frac
     return {"value": batch.num_tokens / t_step, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": (f"decode of {len(seqs)} of {batch.num_seqs} sequences ({frac:.3f} of the keys), "
-                       f"fp64 numpy FP8 reference; step time = full append + sample / key fraction"),
+            "sample": (f"attention of {len(rows)} of {batch.num_tokens} query rows (evenly spaced, {frac:.4f} of "
+                       f"the visible pairs), fp64 numpy FP8 reference; step time = full append + sample / pair "
+                       f"fraction"),
             "sample_seconds": t_sample, "step_seconds_extrapolated": t_step}
-
-
-def run_reference(args):
-    ws, rank, _ = _dist()
-    if rank != 0:
-        return 0
-    batch = W.make_batch(args.workload, seed=args.seed)
-    if args.kv_fp8:
-        _fp8_workload_ok(batch)
-    per = []
-    for i in range(args.warmup + args.steps):
-        r = (cpu_baseline_fp8 if args.kv_fp8 else cpu_baseline)(batch, target_seconds=args.ref_seconds)
-        if i >= args.warmup:
-            per.append(r)
-    step_s = statistics.median(x["step_seconds_extrapolated"] for x in per)
-    value = batch.num_tokens / step_s
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": args.workload, "seed": args.seed,
-                                            "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16"},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": per[0]["cores"], "kind": "oracle",
-                             "sample": per[0]["sample"]},
-            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-            "gpu_launches": 0}
-    print(json.dumps(line), flush=True)
-    return 0
 
 
 def cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds: float = 15.0):
@@ -427,8 +416,9 @@ def run_fnpu_mla_expand(args):
 
 
 def _fp8_workload_ok(batch):
-    if not np.all((batch.query_len == 1) & (batch.phase == 1)):
-        raise SystemExit("--kv-fp8 needs a decode-only workload (qwen_decode)")
+    sh = batch.shape
+    if sh.latent or sh.num_kv_heads != 4 or sh.head_dim_qk != 128 or sh.block_size != 16:
+        raise SystemExit("--kv-fp8 needs the Qwen shape (4 kv heads, d 128, 16-slot blocks)")
 
 
 def run_fnpu(args):
@@ -613,7 +603,7 @@ def main(argv=None):
                     help="MLA prefill without absorption: latent rows expanded into per-head K/V, then MHA "
                          "(latent prefill workloads: mla_prefill)")
     ap.add_argument("--kv-fp8", action="store_true",
-                    help="FP8 (e4m3) KV cache; decode-only workloads (qwen_decode)")
+                    help="FP8 (e4m3) KV cache (Qwen-shaped workloads)")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)  # at least three untimed warm-up steps
     if args.impl == "reference":
