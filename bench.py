@@ -264,6 +264,40 @@ def cpu_baseline_fp8(batch, target_seconds: float = 15.0):
             "sample_seconds": t_sample, "step_seconds_extrapolated": t_step}
 
 
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return 0
+    batch = W.make_batch(args.workload, seed=args.seed)
+    if args.kv_fp8:
+        _fp8_workload_ok(batch)
+    if args.mla_expand:
+        ins = W.mla_expand_inputs(batch, seed=args.seed)
+        slots, bt, _ = W.expanded_layout(batch)
+    per = []
+    for i in range(args.warmup + args.steps):
+        if args.mla_expand:
+            r = cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds=args.ref_seconds)
+        else:
+            r = (cpu_baseline_fp8 if args.kv_fp8 else cpu_baseline)(batch, target_seconds=args.ref_seconds)
+        if i >= args.warmup:
+            per.append(r)
+    step_s = statistics.median(x["step_seconds_extrapolated"] for x in per)
+    value = batch.num_tokens / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": args.workload, "seed": args.seed,
+                                            "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16",
+                                            "path": "mla_expand" if args.mla_expand else "default"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": per[0]["cores"], "kind": "oracle",
+                             "sample": per[0]["sample"]},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds: float = 15.0):
     """Time the fp64 reference of the expanded MLA prefill: the latent append,
     the expansion of every row (numpy), and the C oracle's attention on an
