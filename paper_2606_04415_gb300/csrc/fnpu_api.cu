@@ -46,6 +46,13 @@ struct fnpu_plan {
     fnpu::SeqInfo *d_seqs = nullptr;
     int32_t *d_bt = nullptr;
     fnpu::DecodeItem *d_ditems = nullptr;
+    // FP8 cache with tcgen05 prefill: the prefill sequences' blocks dequantised
+    // to f16 (num_jobs blocks, block table of tbt_width columns) and the
+    // queries in f16, staged before the prefill kernel
+    int32_t num_jobs = 0, tbt_width = 1, num_tblocks = 0;
+    fnpu::Fp8StageJob *d_jobs = nullptr;
+    int32_t *d_tbt = nullptr;
+    void *d_tq = nullptr, *d_tk = nullptr, *d_tv = nullptr;
     fnpu::PrefillItem *d_pitems = nullptr;
     int32_t *d_counters = nullptr;
     int32_t *d_err = nullptr;
@@ -280,6 +287,27 @@ int kernel_support(const fnpu_attn_desc *d, bool has_decode, bool has_prefill) {
 }  // namespace
 }  // namespace fnpu
 
+namespace fnpu {
+namespace {
+// The tcgen05 prefill launch; over the FP8 cache, first the f16 staging of
+// the prefill sequences' blocks and of the queries, and the prefill reads those.
+int launch_prefill(const fnpu_plan *pl, const AttnParams &p, void *stream, int ctas, void *started) {
+    if (!pl->desc.kv_fp8) return launch_prefill_tc(p, stream, ctas, started);
+    const int rc = launch_fp8_stage(p.k_cache, p.v_cache, pl->d_jobs, pl->num_jobs, pl->d_tk, pl->d_tv, p.q, pl->d_tq,
+                                    p.num_tokens * p.num_q_heads * p.head_dim_qk, stream);
+    if (rc != FNPU_OK) return rc;
+    AttnParams pp = p;
+    pp.q = pl->d_tq;
+    pp.k_cache = pl->d_tk;
+    pp.v_cache = pl->d_tv;
+    pp.block_table = pl->d_tbt;
+    pp.bt_stride = pl->tbt_width;
+    pp.num_blocks = pl->num_tblocks;
+    return launch_prefill_tc(pp, stream, ctas, started, true);
+}
+}  // namespace
+}  // namespace fnpu
+
 using namespace fnpu;
 
 extern "C" {
@@ -401,7 +429,7 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                      mla_tc_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_q_heads, desc->num_kv_heads, bs);
     pl->use_dt = !pl->use_mla && decode_tma_supported(desc->head_dim_qk, desc->head_dim_v, desc->num_kv_heads,
                                                       desc->num_q_heads / desc->num_kv_heads, bs);
-    pl->use_tc = !pl->use_mla && !desc->kv_fp8 && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
+    pl->use_tc = !pl->use_mla && !(o.flags & FNPU_PLAN_NO_TCGEN05) &&
                  prefill_tc_supported(desc->head_dim_qk, desc->head_dim_v, bs,
                                       desc->num_q_heads / desc->num_kv_heads);
 
@@ -567,7 +595,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
         int64_t dec_bytes = 0;
         for (const DecodeItem &it : ditems)
             dec_bytes += static_cast<int64_t>(it.key_end - it.key_begin) * desc->num_kv_heads *
-                         (desc->head_dim_qk + desc->head_dim_v) * 2;
+                         (desc->kv_fp8 ? desc->head_dim_qk + desc->head_dim_v + 8
+                                       : (desc->head_dim_qk + desc->head_dim_v) * 2);
         std::vector<int64_t> item_tiles;
         for (const TcUnit &u : tc_units) item_tiles.push_back(u.ntiles + kTcItemCost);
         std::sort(item_tiles.begin(), item_tiles.end(), [](int64_t a, int64_t b) { return a > b; });
@@ -630,6 +659,32 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
             }
         }
     }
+    // FP8 cache, tcgen05 prefill: every prefill sequence's blocks get an f16
+    // copy (its own block-table row over the staged blocks)
+    std::vector<Fp8StageJob> jobs;
+    std::vector<int32_t> tbt;
+    if (desc->kv_fp8 && pl->use_tc && !tc_units.empty()) {
+        std::vector<char> pre(num_seqs, 0);
+        for (const TcUnit &u : tc_units) pre[u.seq] = 1;
+        int32_t tw = 1;
+        for (int32_t s = 0; s < num_seqs; ++s)
+            if (pre[s]) tw = std::max(tw, (context_len[s] + bs - 1) / bs);
+        tbt.assign(static_cast<size_t>(std::max(num_seqs, 1)) * tw, 0);
+        for (int32_t s = 0; s < num_seqs; ++s) {
+            if (!pre[s]) continue;
+            const int32_t nb = (context_len[s] + bs - 1) / bs;
+            for (int32_t j = 0; j < nb; ++j) {
+                const int32_t dst = static_cast<int32_t>(jobs.size());
+                jobs.push_back(Fp8StageJob{dst, block_table[static_cast<int64_t>(s) * block_table_stride + j],
+                                           std::min(bs, context_len[s] - j * bs), 0});
+                tbt[static_cast<size_t>(s) * tw + j] = dst;
+            }
+        }
+        pl->num_jobs = static_cast<int32_t>(jobs.size());
+        pl->tbt_width = tw;
+        pl->num_tblocks = std::max(pl->num_jobs, 1);
+    }
+
     // longest prefill tiles first; decode items longest first as well
     std::stable_sort(pcost.begin(), pcost.end(),
                      [](const std::pair<int64_t, int32_t> &a, const std::pair<int64_t, int32_t> &b) {
@@ -680,6 +735,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
     const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
+    const size_t o_jobs = off; off = align_up(off + sizeof(Fp8StageJob) * std::max<size_t>(jobs.size(), 1), 256);
+    const size_t o_tbt = off; off = align_up(off + sizeof(int32_t) * std::max<size_t>(tbt.size(), 1), 256);
     const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
     const size_t meta_bytes = off;
     // query heads per partial
@@ -690,6 +747,12 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_po = off; off = align_up(off + sizeof(float) * static_cast<size_t>(std::max(parts, 1)) * part_rows * desc->head_dim_v, 256);
     const size_t o_pplse = off; off = align_up(off + sizeof(float) * 256 * static_cast<size_t>(std::max(pparts, 1)), 256);
     const size_t o_ppo = off; off = align_up(off + sizeof(float) * 256 * static_cast<size_t>(std::max(pparts, 1)) * desc->head_dim_v, 256);
+    // FP8 staging: f16 copies of the prefill sequences' blocks and the queries
+    const size_t stage_blk = static_cast<size_t>(bs) * desc->num_kv_heads * desc->head_dim_qk * 2;
+    const size_t o_tk = off; off = align_up(off + (pl->num_jobs ? stage_blk * pl->num_tblocks : 0), 256);
+    const size_t o_tv = off; off = align_up(off + (pl->num_jobs ? stage_blk * pl->num_tblocks : 0), 256);
+    const size_t o_tq = off;
+    off = align_up(off + (pl->num_jobs ? static_cast<size_t>(T) * desc->num_q_heads * desc->head_dim_qk * 2 : 0), 256);
     pl->ws_bytes = off;
 
     if (cudaMalloc(&pl->d_ws, pl->ws_bytes) != cudaSuccess) {
@@ -715,6 +778,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     if (!ditems.empty()) memcpy(h + o_di, ditems.data(), sizeof(DecodeItem) * ditems.size());
     if (!mitems.empty()) memcpy(h + o_mi, mitems.data(), sizeof(MlaItem) * mitems.size());
     if (!mgroups.empty()) memcpy(h + o_mg, mgroups.data(), sizeof(MergeGroup) * mgroups.size());
+    if (!jobs.empty()) memcpy(h + o_jobs, jobs.data(), sizeof(Fp8StageJob) * jobs.size());
+    if (!tbt.empty()) memcpy(h + o_tbt, tbt.data(), sizeof(int32_t) * tbt.size());
     if (!pordered.empty()) memcpy(h + o_pi, pordered.data(), sizeof(PrefillItem) * pordered.size());
 
     uint8_t *d = static_cast<uint8_t *>(pl->d_ws);
@@ -731,6 +796,11 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->d_pcounters = reinterpret_cast<int32_t *>(d + o_pcnt);
     pl->d_ppart_lse = reinterpret_cast<float *>(d + o_pplse);
     pl->d_ppart_o = reinterpret_cast<float *>(d + o_ppo);
+    pl->d_jobs = reinterpret_cast<Fp8StageJob *>(d + o_jobs);
+    pl->d_tbt = reinterpret_cast<int32_t *>(d + o_tbt);
+    pl->d_tk = d + o_tk;
+    pl->d_tv = d + o_tv;
+    pl->d_tq = d + o_tq;
     if (cudaMemcpyAsync(pl->d_ws, pl->h_stage, meta_bytes, cudaMemcpyHostToDevice,
                         static_cast<cudaStream_t>(stream)) != cudaSuccess) {
         cudaGetLastError();
@@ -808,10 +878,11 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
         FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
         const bool green = pl->g_pre != nullptr;  // partitions enforced: no placement order to keep
-        int rc = launch_prefill_tc(p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
+        int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
         if (rc == FNPU_OK) {
             FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, green ? pl->e_fork : pl->e_started, 0));
-            rc = launch_decode_tma(p, pl->s_dec, 3 * (green ? pl->dec_sms : pl->num_sms));
+            const int dctas = 3 * (green ? pl->dec_sms : pl->num_sms);
+            rc = pl->desc.kv_fp8 ? launch_decode_fp8(p, pl->s_dec, dctas) : launch_decode_tma(p, pl->s_dec, dctas);
         }
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
         FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
@@ -823,8 +894,8 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
              : pl->use_dt    ? launch_decode_tma(p, stream, 3 * pl->num_sms)
                              : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
-    if (pl->desc.kv_fp8) return launch_prefill_fp8(p, stream);
-    return pl->use_tc ? launch_prefill_tc(p, stream, pl->num_sms) : launch_prefill_mma(p, stream);
+    if (pl->use_tc) return launch_prefill(pl, p, stream, pl->num_sms, nullptr);
+    return pl->desc.kv_fp8 ? launch_prefill_fp8(p, stream) : launch_prefill_mma(p, stream);
 }
 
 int fnpu_plan_check(const fnpu_plan *pl, void *stream) {

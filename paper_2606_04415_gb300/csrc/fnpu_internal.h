@@ -126,6 +126,14 @@ int launch_kv_append_fp8(const fnpu_attn_desc *d, const void *k_new, const void 
                          void *stream);
 int launch_decode_fp8(const AttnParams &p, void *stream, int max_ctas);
 int launch_prefill_fp8(const AttnParams &p, void *stream);
+// Staging of the FP8 cache for the tcgen05 prefill: job j dequantises source
+// block `src` (valid slots) into f16 block `dst` of k_f16 / v_f16 (plain
+// layout [16 slots][4 heads][128]); the queries are converted bf16 -> f16.
+struct Fp8StageJob {
+    int32_t dst, src, valid, pad;
+};
+int launch_fp8_stage(const void *k_pool, const void *v_pool, const Fp8StageJob *jobs, int32_t num_jobs, void *k_f16,
+                     void *v_f16, const void *q_bf16, void *q_f16, int64_t q_values, void *stream);
 bool decode_fp8_supported(int d_qk, int d_v, int hkv, int group, int block_size);
 int launch_decode_mma(const AttnParams &p, void *stream);
 int launch_decode_tma(const AttnParams &p, void *stream, int max_ctas);
@@ -140,8 +148,9 @@ int mla_tc_keys_per_tile();
 int launch_split_merge(const AttnParams &p, void *stream);
 bool mla_supported(int d_qk, int d_v, int hq, int hkv);
 int mla_heads_per_item();
-// started (a cudaEvent_t, may be null): recorded once every CTA has begun
-int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started = nullptr);
+// started (a cudaEvent_t, may be null): recorded once every CTA has begun;
+// f16: Q, K and V are f16 (d = 128 only), else bf16
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started = nullptr, bool f16 = false);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
 int prefill_tc_rows_per_item(int group);
 int prefill_tc_keys_per_tile();

@@ -258,7 +258,101 @@ __global__ void __launch_bounds__(kThreads, 2) prefill_fp8_kernel(const AttnPara
     }
 }
 
+// One staged block per CTA: the 16 slots x 4 heads x 128 columns of K and of
+// V of a source block, dequantised (code value x row scale, rounded to f16)
+// into the plain cache layout [slot][head][column]; slots past `valid` are
+// zero. K rows: a thread writes 16 columns from the four words that hold them
+// (column 16 k + j at byte 32 c + 4 k + r); V rows: a thread gathers the 8
+// bytes of 8 columns from the transposed block.
+__global__ void __launch_bounds__(128) fp8_dequant_kernel(const uint8_t *__restrict__ kp,
+                                                          const uint8_t *__restrict__ vp,
+                                                          const Fp8StageJob *__restrict__ jobs,
+                                                          uint4 *__restrict__ kd, uint4 *__restrict__ vd) {
+    const Fp8StageJob jb = jobs[blockIdx.x];
+    const uint8_t *kb = kp + static_cast<int64_t>(jb.src) * kBlockBytes;
+    const uint8_t *vb = vp + static_cast<int64_t>(jb.src) * kBlockBytes;
+    const float *ksc = reinterpret_cast<const float *>(kb + kCodeBytes);
+    const float *vsc = reinterpret_cast<const float *>(vb + kCodeBytes);
+    uint4 *ko = kd + static_cast<int64_t>(jb.dst) * (kBs * kHkv * kD / 8);
+    uint4 *vo = vd + static_cast<int64_t>(jb.dst) * (kBs * kHkv * kD / 8);
+    auto scaled = [](uint32_t h2, float sc) {  // f16x2 * sc, rounded to f16x2
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&h2));
+        return pack_f16x2(f.x * sc, f.y * sc);
+    };
+    for (int task = threadIdx.x; task < kBs * kHkv * 8; task += 128) {  // K: row (slot, head) x 16 columns
+        const int row = task >> 3, cg = task & 7;
+        uint4 a = make_uint4(0u, 0u, 0u, 0u), b = a;
+        if ((row >> 2) < jb.valid) {
+            const float sc = ksc[row];
+            uint32_t lo[4], hi[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                e4m3x4_to_f16x2x2(__ldg(reinterpret_cast<const uint32_t *>(kb + row * kD + 32 * c + 4 * cg)), lo[c], hi[c]);
+                lo[c] = scaled(lo[c], sc);
+                hi[c] = scaled(hi[c], sc);
+            }
+            a = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            b = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        }
+        ko[row * (kD / 8) + 2 * cg] = a;
+        ko[row * (kD / 8) + 2 * cg + 1] = b;
+    }
+    for (int task = threadIdx.x; task < kBs * kHkv * 16; task += 128) {  // V: row (slot, head) x 8 columns
+        const int row = task >> 4, cg = task & 15;
+        const int slot = row >> 2, head = row & 3;
+        uint4 out = make_uint4(0u, 0u, 0u, 0u);
+        if (slot < jb.valid) {
+            const float sc = vsc[row];
+            const int vpos = 4 * ((slot & 7) >> 1) + (slot & 1) + 2 * (slot >> 3);
+            const uint8_t *col = vb + head * (kD * kBs) + (8 * cg) * kBs + vpos;
+            uint32_t w0 = 0, w1 = 0;
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                w0 |= static_cast<uint32_t>(__ldg(col + x * kBs)) << (8 * x);
+                w1 |= static_cast<uint32_t>(__ldg(col + (4 + x) * kBs)) << (8 * x);
+            }
+            uint32_t h0, h1, h2, h3;
+            e4m3x4_to_f16x2x2(w0, h0, h1);
+            e4m3x4_to_f16x2x2(w1, h2, h3);
+            out = make_uint4(scaled(h0, sc), scaled(h1, sc), scaled(h2, sc), scaled(h3, sc));
+        }
+        vo[row * (kD / 8) + cg] = out;
+    }
+}
+
+// bf16 -> f16, 8 values per thread and step
+__global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4 *__restrict__ in, uint4 *__restrict__ out,
+                                                          int64_t n8) {
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n8;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const uint4 v = __ldg(in + i);
+        out[i] = make_uint4(bf16x2_to_f16x2(v.x), bf16x2_to_f16x2(v.y), bf16x2_to_f16x2(v.z), bf16x2_to_f16x2(v.w));
+    }
+}
+
 }  // namespace
+
+int launch_fp8_stage(const void *k_pool, const void *v_pool, const Fp8StageJob *jobs, int32_t num_jobs, void *k_f16,
+                     void *v_f16, const void *q_bf16, void *q_f16, int64_t q_values, void *stream) {
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (num_jobs > 0) {
+        fp8_dequant_kernel<<<num_jobs, 128, 0, st>>>(static_cast<const uint8_t *>(k_pool),
+                                                     static_cast<const uint8_t *>(v_pool), jobs,
+                                                     static_cast<uint4 *>(k_f16), static_cast<uint4 *>(v_f16));
+        FNPU_CUDA_TRY(cudaGetLastError());
+    }
+    const int64_t n8 = q_values / 8;
+    if (n8 > 0) {
+        int dev = 0, sms = 148;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const int64_t want = (n8 + 255) / 256;
+        const int grid = static_cast<int>(want < 8LL * sms ? want : 8LL * sms);
+        bf16_to_f16_kernel<<<grid, 256, 0, st>>>(static_cast<const uint4 *>(q_bf16), static_cast<uint4 *>(q_f16), n8);
+        FNPU_CUDA_TRY(cudaGetLastError());
+    }
+    return FNPU_OK;
+}
 
 int launch_prefill_fp8(const AttnParams &p, void *stream) {
     if (p.num_pitems == 0) return FNPU_OK;

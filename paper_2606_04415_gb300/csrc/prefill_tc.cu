@@ -44,6 +44,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "fp8.cuh"
 #include "tc.cuh"
 
 namespace fnpu {
@@ -113,7 +114,9 @@ __device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
     return g;
 }
 
-template <int D>
+// F16: the operands (Q, K, V and P) are f16 instead of bf16 (the FP8 cache's
+// prefill: its codes are dequantised to f16 first)
+template <int D, bool F16>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_tc_kernel(const AttnParams p, const __grid_constant__ TcMaps maps) {
     using Cfg = TcCfg<D>;
@@ -292,8 +295,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // The loop runs with warp-uniform values (passed through __shfl_sync
         // so the compiler keeps them in uniform registers); each tcgen05
         // instruction is issued by one elected lane.
-        constexpr uint32_t idS = tc::idesc_bf16(kRows, kKeys, false);
-        constexpr uint32_t idO = tc::idesc_bf16(kRows, D, true);
+        constexpr uint32_t idS = F16 ? tc::idesc_f16(kRows, kKeys, false) : tc::idesc_bf16(kRows, kKeys, false);
+        constexpr uint32_t idO = F16 ? tc::idesc_f16(kRows, D, true) : tc::idesc_bf16(kRows, D, true);
         const uint32_t utmem = __shfl_sync(0xffffffffu, tmem, 0);
         const uint32_t us_base = __shfl_sync(0xffffffffu, s_base, 0);
         int gk = 0, gv = 0, t = 0, nfix = 0;
@@ -473,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
                         if (j & 1) lacc1 = f2_add(lacc1, f2_pack(p0, p1));
                         else lacc0 = f2_add(lacc0, f2_pack(p0, p1));
-                        pk[j] = pack_bf16x2(p0, p1);
+                        pk[j] = F16 ? pack_f16x2(p0, p1) : pack_bf16x2(p0, p1);
                     }
                     tc::tmem_st16(lane_addr + col_s(w) + 16 * q4, pk);
                 }
@@ -639,7 +642,7 @@ EncodeTiledFn get_encoder() {
 
 // 4-D map over a paged cache [num_blocks, bs, Hkv, d]: box = one block of one
 // kv head, 64 columns wide, 128-byte swizzle.
-bool encode_cache_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, int nblocks) {
+bool encode_cache_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, int nblocks, bool f16) {
     EncodeTiledFn enc = get_encoder();
     if (!enc) return false;
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(hkv), static_cast<cuuint64_t>(bs),
@@ -648,39 +651,41 @@ bool encode_cache_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, 
                              static_cast<cuuint64_t>(bs) * hkv * d * 2};
     cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(bs), 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box, es,
+    return enc(m, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base),
+               dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // 3-D map over q [T, Hq, d]: box = 64 columns x G heads x P positions, so a
 // box lands as the packed (position, head) rows of one Q tile.
-bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, int G, int P) {
+bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, int G, int P, bool f16) {
     EncodeTiledFn enc = get_encoder();
     if (!enc) return false;
     cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(hq), static_cast<cuuint64_t>(T)};
     cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(hq) * d * 2};
     cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(P)};
     cuuint32_t es[3] = {1, 1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+    return enc(m, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base),
+               dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D>
+template <int D, bool F16>
 int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t started) {
     using Cfg = TcCfg<D>;
     TcMaps maps;
-    if (!encode_cache_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
-        !encode_cache_map(&maps.v, p.v_cache, D, p.num_kv_heads, p.block_size, p.num_blocks) ||
-        !encode_q_map(&maps.q, p.q, D, p.num_q_heads, p.num_tokens, p.group, kRows / p.group))
+    if (!encode_cache_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
+        !encode_cache_map(&maps.v, p.v_cache, D, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
+        !encode_q_map(&maps.q, p.q, D, p.num_q_heads, p.num_tokens, p.group, kRows / p.group, F16))
         return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
-    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D, F16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmemBytes));
-    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout,
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D, F16>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                        cudaSharedmemCarveoutMaxShared));
     const int grid = p.num_pitems < max_ctas ? p.num_pitems : max_ctas;
-    FNPU_CUDA_TRY(launch_ex(prefill_tc_kernel<D>, grid, kThreads, Cfg::kSmemBytes, st, false, started, p, maps));
+    FNPU_CUDA_TRY(launch_ex(prefill_tc_kernel<D, F16>, grid, kThreads, Cfg::kSmemBytes, st, false, started, p, maps));
     return FNPU_OK;
 }
 
@@ -697,12 +702,14 @@ int prefill_tc_rows_per_item(int group) { return 2 * (kRows / group); }
 // keys per K/V tile (the unit of the planner's key splits)
 int prefill_tc_keys_per_tile() { return kKeys; }
 
-int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started) {
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started, bool f16) {
     if (p.num_pitems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaEvent_t ev = static_cast<cudaEvent_t>(started);
+    if (f16) return p.head_dim_qk == 128 ? launch_tc<128, true>(p, st, max_ctas, ev) : FNPU_EUNSUPPORTED;
     switch (p.head_dim_qk) {
-        case 64: return launch_tc<64>(p, st, max_ctas, static_cast<cudaEvent_t>(started));
-        case 128: return launch_tc<128>(p, st, max_ctas, static_cast<cudaEvent_t>(started));
+        case 64: return launch_tc<64, false>(p, st, max_ctas, ev);
+        case 128: return launch_tc<128, false>(p, st, max_ctas, ev);
         default: return FNPU_EUNSUPPORTED;
     }
 }

@@ -267,8 +267,13 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo_byt
     d |= static_cast<uint64_t>(2) << 61;  // SWIZZLE_128B
     return d;
 }
-// Instruction descriptor of kind::f16 with bf16 A and B and an fp32 D.
-// A is K-major (or in tensor memory); B is K-major or MN-major.
+// Instruction descriptor of kind::f16 with f16 A and B (format fields 0) and
+// an fp32 D. A is K-major (or in tensor memory); B is K-major or MN-major.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool b_mn_major) {
+    return (1u << 4) | ((b_mn_major ? 1u : 0u) << 16) | (static_cast<uint32_t>(N >> 3) << 17) |
+           (static_cast<uint32_t>(M >> 4) << 24);
+}
+// The same with bf16 A and B (format fields 1).
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
            (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);

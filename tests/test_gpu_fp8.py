@@ -57,11 +57,11 @@ def _reference_pools(batch, init, seqs=None):
     return F8.kv_append(kp, vp, kn, vn, sm, 4)
 
 
-def _run(batch, seed=0, split=0, check_pools=True):
+def _run(batch, seed=0, split=0, check_pools=True, flags=0, share=0):
     import paper_2606_04415_gb300 as fnpu
     from paper_2606_04415_gb300.step import DeviceStep
     init = W.stale_pool_bytes(batch.num_blocks * F8.block_bytes(4), seed)
-    st = DeviceStep(batch, opts=fnpu.PlanOpts(split, 0, 0, 0), kv_fp8=True, pool_init=init)
+    st = DeviceStep(batch, opts=fnpu.PlanOpts(split, share, 0, flags), kv_fp8=True, pool_init=init)
     st.run()
     assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK and fnpu.check() == fnpu.FNPU_OK
     out, lse = st.results()
@@ -181,15 +181,32 @@ def test_fp8_plan_reuse_runs_repeatedly():
     _compare(batch, o2, l2, kp, vp)
 
 
+@pytest.mark.parametrize("flags", [0, 2])
 @pytest.mark.parametrize("hq", [28, 32])
-def test_fp8_mixed_step_prefill_and_decode(hq):
+def test_fp8_mixed_step_prefill_and_decode(hq, flags):
     """Prefill chunks on prefixes (64 rows on none, 130 on 170), a 3-token
     decode (the prefill queue) and one-token decodes (one of 2049 keys) over
-    the FP8 cache: the prefill rows run on the f16 mma.sync FP8 prefill kernel,
-    the decodes on the FP8 decode kernel; all rows against the reference."""
+    the FP8 cache: the prefill rows on the tcgen05 kernel over f16-staged blocks
+    (flags 0) or on the f16 mma.sync FP8 kernel (FNPU_PLAN_NO_TCGEN05), the
+    decodes on the FP8 decode kernel; all rows against the reference."""
     batch = _batch([64, 500, 300, 200, 2049], hq=hq, seed=7, ql=[64, 1, 130, 3, 1], phase=[0, 1, 0, 1, 1])
-    _, out, lse, kp, vp = _run(batch, seed=7)
+    _, out, lse, kp, vp = _run(batch, seed=7, flags=flags)
     _compare(batch, out, lse, kp, vp)
+
+
+@pytest.mark.parametrize("share", [0, 20])
+def test_fp8_colocated_and_separate_launches_agree(share):
+    """A co-located FP8 step (prefill on tcgen05 over the staged blocks beside
+    the FP8 decode kernel) at the planner's and a fixed decode share, and the
+    same step as separate launches: parity against the reference, and the two
+    launch modes within rounding of each other."""
+    import paper_2606_04415_gb300 as fnpu
+    batch = _batch([1000, 700, 64, 3000, 129, 900], hq=28, seed=9, ql=[300, 1, 64, 1, 1, 1],
+                   phase=[0, 1, 0, 1, 1, 1])
+    st, out, lse, kp, vp = _run(batch, seed=9, share=share)
+    _compare(batch, out, lse, kp, vp)
+    st2, out2, lse2, _, _ = _run(batch, seed=9, flags=fnpu.PLAN_SEPARATE_LAUNCHES, check_pools=False)
+    assert np.abs(out - out2).max() <= 1e-2 and np.abs(lse - lse2).max() <= 1e-3
 
 
 def test_fp8_colocated_workload_sampled_rows():
