@@ -76,9 +76,10 @@ typedef struct {
  * Sec. 3.3); one-byte values halve them. The paper quantises its DeepSeek-R1
  * deployment to 8 bits (Sec. 4.1) but gives no cache format; this is the
  * library's. Supported for split K/V with Hkv = 4, d_qk = d_v = 128,
- * block_size = 16, Hq / Hkv <= 8 (decode, prefill and mixed plans; a mixed
- * plan launches its decode and prefill kernels one after the other);
- * anything else returns FNPU_EUNSUPPORTED.
+ * block_size = 16, Hq / Hkv <= 8 (decode, prefill and mixed plans; the plan
+ * stages an f16 copy of its prefill sequences' blocks and queries for the
+ * tensor-core prefill, so values must lie within the f16 range); anything
+ * else returns FNPU_EUNSUPPORTED.
  *   Quantisation, per stored row (one slot, one kv head, 128 values):
  *     scale = amax |x| / 448 in fp32 (1 for a zero row), code = the e4m3 value
  *     nearest to x / scale (fp32 quotient; ties to the even code; magnitudes
