@@ -1,6 +1,12 @@
-// Prefill attention over the FP8 (e4m3) KV cache, on f16 mma.sync.
+// Prefill over the FP8 (e4m3) KV cache.
 //
-// The chunk rows of a mixed step whose cache is stored in the library's FP8
+// Two ways. By default the plan stages an f16 copy of its prefill sequences'
+// blocks (fp8_dequant_kernel: code value x row scale, rounded once to f16)
+// and of the queries, and the tcgen05 prefill kernel runs on those with f16
+// operands. With FNPU_PLAN_NO_TCGEN05, prefill_fp8_kernel below reads the
+// codes directly on f16 mma.sync.
+//
+// prefill_fp8_kernel: the chunk rows of a mixed step whose cache is stored in the library's FP8
 // format (include/fnpu.h; Hkv = 4, d = 128, 16-slot blocks). The structure is
 // the mma.sync prefill kernel's: one CTA computes 64 query rows of one query
 // head, four warps own 16 rows each, 64-key tiles (four blocks) are staged
