@@ -268,8 +268,9 @@ __global__ void __launch_bounds__(kThreads, 2) prefill_fp8_kernel(const AttnPara
 // V of a source block, dequantised (code value x row scale, rounded to f16)
 // into the plain cache layout [slot][head][column]; slots past `valid` are
 // zero. K rows: a thread writes 16 columns from the four words that hold them
-// (column 16 k + j at byte 32 c + 4 k + r); V rows: a thread gathers the 8
-// bytes of 8 columns from the transposed block.
+// (column 16 k + j at byte 32 c + 4 k + r); V: a thread reads one stored
+// column (16 slots, 16 bytes; a warp reads 512 contiguous bytes) and writes
+// its 16 values into their rows (a warp writes 64 contiguous bytes a row).
 __global__ void __launch_bounds__(128) fp8_dequant_kernel(const uint8_t *__restrict__ kp,
                                                           const uint8_t *__restrict__ vp,
                                                           const Fp8StageJob *__restrict__ jobs,
@@ -303,26 +304,26 @@ __global__ void __launch_bounds__(128) fp8_dequant_kernel(const uint8_t *__restr
         ko[row * (kD / 8) + 2 * cg] = a;
         ko[row * (kD / 8) + 2 * cg + 1] = b;
     }
-    for (int task = threadIdx.x; task < kBs * kHkv * 16; task += 128) {  // V: row (slot, head) x 8 columns
-        const int row = task >> 4, cg = task & 15;
-        const int slot = row >> 2, head = row & 3;
-        uint4 out = make_uint4(0u, 0u, 0u, 0u);
-        if (slot < jb.valid) {
-            const float sc = vsc[row];
-            const int vpos = 4 * ((slot & 7) >> 1) + (slot & 1) + 2 * (slot >> 3);
-            const uint8_t *col = vb + head * (kD * kBs) + (8 * cg) * kBs + vpos;
-            uint32_t w0 = 0, w1 = 0;
+    __half *vh = reinterpret_cast<__half *>(vo);
+    for (int task = threadIdx.x; task < kHkv * kD; task += 128) {  // V: one stored column (head, d), 16 slots
+        const int head = task >> 7, d = task & (kD - 1);
+        const uint4 w = __ldg(reinterpret_cast<const uint4 *>(vb + head * (kD * kBs) + d * kBs));
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-            for (int x = 0; x < 4; ++x) {
-                w0 |= static_cast<uint32_t>(__ldg(col + x * kBs)) << (8 * x);
-                w1 |= static_cast<uint32_t>(__ldg(col + (4 + x) * kBs)) << (8 * x);
+        for (int c = 0; c < 4; ++c) {  // word c: slots 2c, 2c + 1 (lo) and 2c + 8, 2c + 9 (hi)
+            uint32_t lo, hi;
+            e4m3x4_to_f16x2x2(ws[c], lo, hi);
+            const float2 fl = __half22float2(*reinterpret_cast<const __half2 *>(&lo));
+            const float2 fh = __half22float2(*reinterpret_cast<const __half2 *>(&hi));
+            const int sl[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+            const float f[4] = {fl.x, fl.y, fh.x, fh.y};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int o = sl[e];
+                vh[(o * kHkv + head) * kD + d] =
+                    __float2half_rn(o < jb.valid ? f[e] * vsc[o * kHkv + head] : 0.f);
             }
-            uint32_t h0, h1, h2, h3;
-            e4m3x4_to_f16x2x2(w0, h0, h1);
-            e4m3x4_to_f16x2x2(w1, h2, h3);
-            out = make_uint4(scaled(h0, sc), scaled(h1, sc), scaled(h2, sc), scaled(h3, sc));
         }
-        vo[row * (kD / 8) + cg] = out;
     }
 }
 
