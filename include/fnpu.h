@@ -168,7 +168,8 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs,
 
 /*
  * Attention for every query of the planned step. q, k_cache, v_cache, out,
- * lse are device pointers in the layouts above (v_cache NULL for latent).
+ * lse are device pointers in the layouts above (v_cache NULL for latent;
+ * with kv_fp8 = 1, k_cache and v_cache are the FP8 byte pools).
  * Enqueues the work on `stream` and returns without synchronising. Runs of
  * one plan must not overlap on the GPU (they share the plan's split scratch).
  * Errors: FNPU_EINVAL (NULL pointers), FNPU_ECUDA (launch failure).
