@@ -229,3 +229,16 @@ def test_fp8_colocated_workload_sampled_rows():
     rows = sorted({0, 1, 63, 64, 65, 127, 1023, 1024, 2047} | set(rng.integers(0, 2048, 10).tolist()))
     tokens = np.asarray(rows + [int(batch.query_start[s]) for s in dec], np.int64)
     _compare(batch, out, lse, kp, vp, tokens=tokens)
+
+
+def test_fp8_colocated_in_green_context_partitions():
+    """A co-located FP8 step with the SM split enforced by green contexts (the
+    staging kernels and the tcgen05 prefill in the prefill partition, the FP8
+    decode in the decode partition): parity against the reference."""
+    import paper_2606_04415_gb300 as fnpu
+    batch = _batch([1000, 700, 64, 3000, 129, 900], hq=28, seed=10, ql=[300, 1, 64, 1, 1, 1],
+                   phase=[0, 1, 0, 1, 1, 1])
+    st, out, lse, kp, vp = _run(batch, seed=10, flags=fnpu.PLAN_GREEN_CONTEXTS, share=20)
+    _compare(batch, out, lse, kp, vp)
+    pre, dec = fnpu.plan_phase_ms(st.plan)
+    assert pre > 0 and dec > 0
