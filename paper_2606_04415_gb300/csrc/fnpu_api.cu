@@ -935,7 +935,7 @@ int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_
     if (decode_items) *decode_items = pl->num_ditems;
     if (launches_per_run)
         *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0) + (pl->num_mgroups > 0) +
-                            (pl->num_jobs > 0 ? 2 : 0);  // FP8 staging: blocks and queries to f16
+                            (pl->num_jobs > 0 ? 1 : 0);  // FP8 staging: blocks and queries to f16
     if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_bytes);
     return FNPU_OK;
 }

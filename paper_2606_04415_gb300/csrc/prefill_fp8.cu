@@ -1,7 +1,7 @@
 // Prefill over the FP8 (e4m3) KV cache.
 //
 // Two ways. By default the plan stages an f16 copy of its prefill sequences'
-// blocks (fp8_dequant_kernel: code value x row scale, rounded once to f16)
+// blocks (fp8_stage_kernel: code value x row scale, rounded once to f16)
 // and of the queries, and the tcgen05 prefill kernel runs on those with f16
 // operands. With FNPU_PLAN_NO_TCGEN05, prefill_fp8_kernel below reads the
 // codes directly on f16 mma.sync.
@@ -264,18 +264,16 @@ __global__ void __launch_bounds__(kThreads, 2) prefill_fp8_kernel(const AttnPara
     }
 }
 
-// One staged block per CTA: the 16 slots x 4 heads x 128 columns of K and of
+// One staged block (a CTA): the 16 slots x 4 heads x 128 columns of K and of
 // V of a source block, dequantised (code value x row scale, rounded to f16)
 // into the plain cache layout [slot][head][column]; slots past `valid` are
 // zero. K rows: a thread writes 16 columns from the four words that hold them
 // (column 16 k + j at byte 32 c + 4 k + r); V: a thread reads one stored
 // column (16 slots, 16 bytes; a warp reads 512 contiguous bytes) and writes
 // its 16 values into their rows (a warp writes 64 contiguous bytes a row).
-__global__ void __launch_bounds__(128) fp8_dequant_kernel(const uint8_t *__restrict__ kp,
-                                                          const uint8_t *__restrict__ vp,
-                                                          const Fp8StageJob *__restrict__ jobs,
-                                                          uint4 *__restrict__ kd, uint4 *__restrict__ vd) {
-    const Fp8StageJob jb = jobs[blockIdx.x];
+__device__ __forceinline__ void fp8_dequant_block(const uint8_t *__restrict__ kp, const uint8_t *__restrict__ vp,
+                                                  const Fp8StageJob jb, uint4 *__restrict__ kd,
+                                                  uint4 *__restrict__ vd) {
     const uint8_t *kb = kp + static_cast<int64_t>(jb.src) * kBlockBytes;
     const uint8_t *vb = vp + static_cast<int64_t>(jb.src) * kBlockBytes;
     const float *ksc = reinterpret_cast<const float *>(kb + kCodeBytes);
@@ -327,13 +325,22 @@ __global__ void __launch_bounds__(128) fp8_dequant_kernel(const uint8_t *__restr
     }
 }
 
-// bf16 -> f16, 8 values per thread and step
-__global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4 *__restrict__ in, uint4 *__restrict__ out,
-                                                          int64_t n8) {
-    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n8;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const uint4 v = __ldg(in + i);
-        out[i] = make_uint4(bf16x2_to_f16x2(v.x), bf16x2_to_f16x2(v.y), bf16x2_to_f16x2(v.z), bf16x2_to_f16x2(v.w));
+// The staging in one launch: CTAs below num_jobs dequantise one block each,
+// the others convert the queries bf16 -> f16 (8 values per thread and step).
+__global__ void __launch_bounds__(128) fp8_stage_kernel(const uint8_t *__restrict__ kp, const uint8_t *__restrict__ vp,
+                                                        const Fp8StageJob *__restrict__ jobs, int32_t num_jobs,
+                                                        uint4 *__restrict__ kd, uint4 *__restrict__ vd,
+                                                        const uint4 *__restrict__ qin, uint4 *__restrict__ qout,
+                                                        int64_t n8) {
+    if (static_cast<int32_t>(blockIdx.x) < num_jobs) {
+        fp8_dequant_block(kp, vp, jobs[blockIdx.x], kd, vd);
+        return;
+    }
+    const int64_t nq = static_cast<int64_t>(gridDim.x) - num_jobs;
+    for (int64_t i = (static_cast<int64_t>(blockIdx.x) - num_jobs) * blockDim.x + threadIdx.x; i < n8;
+         i += nq * blockDim.x) {
+        const uint4 v = __ldg(qin + i);
+        qout[i] = make_uint4(bf16x2_to_f16x2(v.x), bf16x2_to_f16x2(v.y), bf16x2_to_f16x2(v.z), bf16x2_to_f16x2(v.w));
     }
 }
 
@@ -341,23 +348,18 @@ __global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4 *__restric
 
 int launch_fp8_stage(const void *k_pool, const void *v_pool, const Fp8StageJob *jobs, int32_t num_jobs, void *k_f16,
                      void *v_f16, const void *q_bf16, void *q_f16, int64_t q_values, void *stream) {
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (num_jobs > 0) {
-        fp8_dequant_kernel<<<num_jobs, 128, 0, st>>>(static_cast<const uint8_t *>(k_pool),
-                                                     static_cast<const uint8_t *>(v_pool), jobs,
-                                                     static_cast<uint4 *>(k_f16), static_cast<uint4 *>(v_f16));
-        FNPU_CUDA_TRY(cudaGetLastError());
-    }
     const int64_t n8 = q_values / 8;
-    if (n8 > 0) {
-        int dev = 0, sms = 148;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        const int64_t want = (n8 + 255) / 256;
-        const int grid = static_cast<int>(want < 8LL * sms ? want : 8LL * sms);
-        bf16_to_f16_kernel<<<grid, 256, 0, st>>>(static_cast<const uint4 *>(q_bf16), static_cast<uint4 *>(q_f16), n8);
-        FNPU_CUDA_TRY(cudaGetLastError());
-    }
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (n8 + 127) / 128;
+    const int64_t qctas = want < 4LL * sms ? want : 4LL * sms;
+    if (num_jobs + qctas == 0) return FNPU_OK;
+    fp8_stage_kernel<<<static_cast<int>(num_jobs + qctas), 128, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint8_t *>(k_pool), static_cast<const uint8_t *>(v_pool), jobs, num_jobs,
+        static_cast<uint4 *>(k_f16), static_cast<uint4 *>(v_f16), static_cast<const uint4 *>(q_bf16),
+        static_cast<uint4 *>(q_f16), n8);
+    FNPU_CUDA_TRY(cudaGetLastError());
     return FNPU_OK;
 }
 
