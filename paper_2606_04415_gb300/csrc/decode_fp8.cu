@@ -31,10 +31,7 @@
 //     to zero in registers (stale slots may hold NaN codes).
 // Every mbarrier wait is bounded and raises the plan's error flag on timeout.
 #include <cuda_fp16.h>
-#include <cuda_fp8.h>
 #include <math.h>
-
-#include <mutex>
 
 #include "common.cuh"
 #include "fp8.cuh"
@@ -432,30 +429,11 @@ __global__ void __launch_bounds__(kThreads, 3)
     }
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
-                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
-                                  CUtensorMapFloatOOBfill);
-
-EncodeTiledFn fp8_encoder() {
-    static std::once_flag once;
-    static EncodeTiledFn fn = nullptr;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    });
-    return fn;
-}
-
 // K codes: bytes [block][slot][head][128] with the slot dimension listed
 // before the head dimension, so that a box (128 bytes, 16 slots, 4 heads, 1
 // block) lands head-major; 128-byte swizzle keyed by the slot.
 bool encode_k_map(CUtensorMap *m, const void *base, int nblocks) {
-    EncodeTiledFn enc = fp8_encoder();
+    EncodeTiledFn enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(kD), kKeys, kHkv, static_cast<cuuint64_t>(nblocks)};
     cuuint64_t strides[3] = {kHkv * kD, kD, kBlockBytes};

@@ -36,8 +36,6 @@
 // Every mbarrier wait is bounded and raises the plan's error flag on timeout.
 #include <math.h>
 
-#include <mutex>
-
 #include "common.cuh"
 #include "tc.cuh"
 
@@ -482,30 +480,11 @@ __global__ void __launch_bounds__(32 * kMergeWarps) split_merge_kernel(const Att
     if (lane == 0) p.lse[static_cast<int64_t>(mg.token) * Hq + h] = (M + log2f(L)) * kLn2;
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
-                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
-                                  CUtensorMapFloatOOBfill);
-
-EncodeTiledFn dt_encoder() {
-    static std::once_flag once;
-    static EncodeTiledFn fn = nullptr;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    });
-    return fn;
-}
-
 // 4-D map over a paged cache [num_blocks, bs, Hkv, d] with the slot dimension
 // listed before the kv-head dimension: a box (64 columns, 16 slots, Hkv heads,
 // 1 block) lands in shared memory head-major.
 bool encode_slot_major_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, int nblocks) {
-    EncodeTiledFn enc = dt_encoder();
+    EncodeTiledFn enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(bs), static_cast<cuuint64_t>(hkv),
                           static_cast<cuuint64_t>(nblocks)};

@@ -243,6 +243,24 @@ std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int
     return best;
 }
 
+}  // namespace
+
+EncodeTiledFn tensor_map_encoder() {
+    static std::once_flag once;
+    static EncodeTiledFn fn = nullptr;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+namespace {
+
 bool shape_ok(const fnpu_attn_desc *d, int *status) {
     *status = FNPU_EINVAL;
     if (!d) return false;

@@ -1,6 +1,7 @@
 // Internal structures shared between the host planner and the kernels.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -102,6 +103,14 @@ struct AttnParams {
     int32_t *err;           // device error flag of the plan
     int32_t *sched;         // persistent work queues: [0..1] prefill, [2..3] decode (next item, finished CTAs)
 };
+
+// cuTensorMapEncodeTiled, looked up once through the runtime's driver entry
+// point (the library does not link the driver library); null if unavailable.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
 
 // Record a failed CUDA call for fnpu_last_cuda_error(); returns FNPU_ECUDA.
 int cuda_fail(cudaError_t e, const char *where);

@@ -27,8 +27,6 @@
 // 2^8) happens while no product is writing O.
 #include <math.h>
 
-#include <mutex>
-
 #include "common.cuh"
 #include "tc.cuh"
 
@@ -367,30 +365,11 @@ __global__ void __launch_bounds__(kThreads, 1) mla_tc_kernel(const AttnParams p,
     }
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
-                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
-                                  CUtensorMapFloatOOBfill);
-
-EncodeTiledFn mla_encoder() {
-    static std::once_flag once;
-    static EncodeTiledFn fn = nullptr;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    });
-    return fn;
-}
-
 // 3-D map, 64 columns by `rows` rows by 1, 128-byte swizzle: over the latent
 // cache [blocks, bs, 576] (box = one block) or over Q [T, 128, 576] (box = one
 // token's 128 heads).
 bool encode_rows_map(CUtensorMap *m, const void *base, int64_t row_stride_elems, int rows, int64_t outer) {
-    EncodeTiledFn enc = mla_encoder();
+    EncodeTiledFn enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[3] = {static_cast<cuuint64_t>(kDq), static_cast<cuuint64_t>(rows), static_cast<cuuint64_t>(outer)};
     cuuint64_t strides[2] = {static_cast<cuuint64_t>(row_stride_elems) * 2,

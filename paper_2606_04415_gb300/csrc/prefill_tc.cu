@@ -41,8 +41,6 @@
 // the CTA drains its tensor-core work, frees its tensor memory and exits.
 #include <math.h>
 
-#include <mutex>
-
 #include "common.cuh"
 #include "fp8.cuh"
 #include "tc.cuh"
@@ -621,29 +619,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
-                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
-                                  CUtensorMapFloatOOBfill);
-
-EncodeTiledFn get_encoder() {
-    static std::once_flag once;
-    static EncodeTiledFn fn = nullptr;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    });
-    return fn;
-}
-
 // 4-D map over a paged cache [num_blocks, bs, Hkv, d]: box = one block of one
 // kv head, 64 columns wide, 128-byte swizzle.
 bool encode_cache_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, int nblocks, bool f16) {
-    EncodeTiledFn enc = get_encoder();
+    EncodeTiledFn enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(hkv), static_cast<cuuint64_t>(bs),
                           static_cast<cuuint64_t>(nblocks)};
@@ -660,7 +639,7 @@ bool encode_cache_map(CUtensorMap *m, const void *base, int d, int hkv, int bs, 
 // 3-D map over q [T, Hq, d]: box = 64 columns x G heads x P positions, so a
 // box lands as the packed (position, head) rows of one Q tile.
 bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, int G, int P, bool f16) {
-    EncodeTiledFn enc = get_encoder();
+    EncodeTiledFn enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(hq), static_cast<cuuint64_t>(T)};
     cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(hq) * d * 2};
