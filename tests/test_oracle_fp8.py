@@ -86,14 +86,16 @@ def test_pack_unpack_round_trip_and_append():
     back = fp8.unpack_pools(kp, vp, hkv)
     for a, b in zip(back, (kc, ks, vc, vs)):
         assert np.array_equal(a, b)
-    new_k = _bf16(rng.standard_normal((3, hkv, 128)))
-    new_v = _bf16(rng.standard_normal((3, hkv, 128)))
-    slots = np.array([17, -1, 79], np.int64)
+    new_k = _bf16(rng.standard_normal((4, hkv, 128)))
+    new_v = _bf16(rng.standard_normal((4, hkv, 128)))
+    slots = np.array([17, -1, 79, 0], np.int64)
     kp2, vp2 = fp8.kv_append(kp, vp, new_k, new_v, slots, hkv)
     k2, ks2, v2, vs2 = fp8.unpack_pools(kp2, vp2, hkv)
     qk, sk = fp8.quantize_rows(new_k)
+    qv, sv = fp8.quantize_rows(new_v)
     assert np.array_equal(k2[1, 1], qk[0]) and np.array_equal(ks2[4, 15], sk[2])
-    assert np.array_equal(k2[0], kc[0]) and np.array_equal(v2[2], vc[2])   # untouched blocks
+    assert np.array_equal(k2[0, 0], qk[3]) and np.array_equal(v2[0, 0], qv[3]) and vs2[0, 0, 1] == sv[3, 1]
+    assert np.array_equal(k2[3], kc[3]) and np.array_equal(v2[2], vc[2])   # untouched blocks
 
 
 def test_decode_attention_closed_forms():
