@@ -479,6 +479,17 @@ def run_fnpu(args):
         st = DeviceStep(batch, opts=opts, device=str(dev), kv_fp8=True, pool_init=init)
     else:
         st = DeviceStep(batch, opts=opts, device=str(dev))
+    # the plan (host: validation, work lists, workspace, one async upload),
+    # timed apart from the step: median host time of a few plans of the batch
+    torch.cuda.synchronize(dev)
+    plan_ms = []
+    for _ in range(5):
+        t0 = time.perf_counter()
+        extra = fnpu.mixed_attn_plan(st.desc, batch.query_len, batch.context_len, batch.phase, batch.block_table,
+                                     opts=opts)
+        plan_ms.append((time.perf_counter() - t0) * 1e3)
+        extra.destroy()
+    torch.cuda.synchronize(dev)
     info = st.plan.info()
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
@@ -589,7 +600,8 @@ def run_fnpu(args):
         "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T,
                    "num_seqs": batch.num_seqs, "prefill_ctx": int(batch.context_len[0]),
                    "flops": F, "bytes": work["bytes"], "l2": "flushed between timed steps (512 MB write, then 256 MB read)",
-                   "plan": info, "dispatch": args.dispatch, "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16"},
+                   "plan": info, "plan_host_ms": round(statistics.median(plan_ms), 3),
+                   "dispatch": args.dispatch, "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16"},
         "roofline": roof,
         "roofline_step_frac": {"burst": step_roof / (step_ms * 1e-3),
                                "sustained": step_roof_sus / (step_ms * 1e-3),
