@@ -49,9 +49,9 @@ L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 # summaries with the commands are under profiles/. Set to None for a
 # workload whose kernels change until they are captured again.
 NCU_TRAFFIC = {
-    "qwen_coloc": 472.3e6,       # prefill_tc 33.3 MB + decode_tma 437.7 MB read + 1.3 MB write
-    "qwen_decode": 308.7e6,      # decode_tma 308.15 MB read + 0.55 MB write
-    "qwen_decode_fp8": 159.5e6,  # decode_fp8 159.16 MB read + 0.37 MB write
+    "qwen_coloc": 472.4e6,       # prefill_tc 33.3 MB + decode_tma 437.7 MB read + 1.4 MB write
+    "qwen_decode": 308.9e6,      # decode_tma 308.15 MB read + 0.7 MB write
+    "qwen_decode_fp8": 159.6e6,  # decode_fp8 159.16 MB read + 0.4 MB write
 }
 
 
