@@ -71,6 +71,7 @@ __global__ void __launch_bounds__(kThreads, 2) prefill_mma_kernel(const AttnPara
         const uint32_t sK = sKV + stage * Cfg::kStageBytes;
         const uint32_t sV = sK + Cfg::kKBytes;
         if constexpr (DQ == DV) {  // one slot lookup for a K and a V chunk
+            static_assert(Cfg::kQChunks == Cfg::kVChunks, "equal row widths");
 #pragma unroll 4
             for (int i = tid; i < kKeys * Cfg::kQChunks; i += kThreads) {
                 const int row = i / Cfg::kQChunks, ch = i % Cfg::kQChunks;
