@@ -119,3 +119,39 @@ def test_attention_oracle_on_expanded_rows_matches_brute_force():
                 assert np.allclose(out[t, h], p @ vf[base:base + pos + 1, h] / p.sum(), atol=1e-12)
                 assert np.isclose(lse[t, h], x.max() + np.log(p.sum()), atol=1e-12)
             t += 1
+
+
+def test_expanded_path_equals_the_c_latent_oracle_with_selection_weights():
+    """With W_UK[h] selecting latent columns 64h .. 64h + 127 and W_UV[h]
+    columns 128 + 32h .. 255 + 32h, every expanded value and the absorbed
+    query [W_UK[h] q_nope, q_rope] are exact in bf16, so the expanded
+    reference (this module + the C oracle at 192 / 128, one kv head per head)
+    must equal the C oracle's latent attention (576 / 512, one latent head) with
+    that query, its output columns selected by W_UV[h]: two independent paths."""
+    rng = np.random.default_rng(9)
+    H = 4
+    sh = W.Shape(H, 1, 576, 512, 64, True)
+    batch = W.build_batch(sh, [7, 1, 20], [30, 90, 20], [0, 0, 0], rng, name="mla_sel")
+    wk = np.zeros((H, 512, 128), np.float32)
+    wv = np.zeros((H, 512, 128), np.float32)
+    for h in range(H):
+        wk[h, 64 * h + np.arange(128), np.arange(128)] = 1.0
+        wv[h, 128 + 32 * h + np.arange(128), np.arange(128)] = 1.0
+    wk, wv = W.f32_to_bf16_bits(wk), W.f32_to_bf16_bits(wv)
+    q = W.f32_to_bf16_bits(rng.standard_normal((batch.num_tokens, H, 192)).astype(np.float32))
+    lat = oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping)
+    slots, bt, _ = W.expanded_layout(batch)
+    kb, vb = X.expand(lat, slots, wk, wv)
+    scale = 1.0 / np.sqrt(192)
+    out_e, lse_e = oracle.attention(batch.query_len, batch.context_len, bt, q, kb, vb, num_q_heads=H,
+                                    num_kv_heads=H, head_dim_qk=192, head_dim_v=128, block_size=16, scale=scale)
+    q_abs = np.zeros((batch.num_tokens, H, 576), np.uint16)
+    for h in range(H):
+        q_abs[:, h, 64 * h:64 * h + 128] = q[:, h, :128]
+        q_abs[:, h, 512:] = q[:, h, 128:]
+    out_l, lse_l = oracle.attention(batch.query_len, batch.context_len, batch.block_table, q_abs, lat, None,
+                                    num_q_heads=H, num_kv_heads=1, head_dim_qk=576, head_dim_v=512, block_size=64,
+                                    latent=True, scale=scale)
+    for h in range(H):
+        assert np.abs(out_e[:, h] - out_l[:, h, 128 + 32 * h:256 + 32 * h]).max() < 1e-12
+    assert np.abs(lse_e - lse_l).max() < 1e-12
