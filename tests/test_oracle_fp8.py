@@ -183,3 +183,17 @@ def test_mixed_step_matches_the_bf16_oracle_when_every_scale_is_one():
     tok = np.array([0, 19, 21, 23, 24])
     o2, l2 = fp8.attention(ql, cl, bt, q, kp, vp, num_q_heads=hq, num_kv_heads=hkv, tokens=tok)
     assert np.array_equal(o2, out[tok]) and np.array_equal(l2, lse[tok])
+
+
+def test_worked_example_from_the_golden_file():
+    """tests/golden/fp8_row_example.txt: a row quantised by hand."""
+    import os
+    path = os.path.join(os.path.dirname(__file__), "golden", "fp8_row_example.txt")
+    lines = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
+    want_scale = float(lines[0][1])
+    want_codes = [int(c) for c in lines[1][1:]]
+    x = np.zeros(128, np.float32)
+    x[:5] = [3.5, -1.75, 0.0078125, 5.25, 0.001]
+    codes, scale = fp8.quantize_rows(_bf16(x)[None])
+    assert scale[0] == np.float32(want_scale)
+    assert codes[0, :5].tolist() == want_codes and not codes[0, 5:].any()
