@@ -197,3 +197,28 @@ def test_worked_example_from_the_golden_file():
     codes, scale = fp8.quantize_rows(_bf16(x)[None])
     assert scale[0] == np.float32(want_scale)
     assert codes[0, :5].tolist() == want_codes and not codes[0, 5:].any()
+
+
+def test_zero_keys_give_the_mean_of_the_dequantised_values():
+    """K codes all zero: every score is 0, the weights are uniform, so O is the
+    mean of the visible dequantised values (each row with its own V scale) and
+    LSE = ln(pos + 1); for decodes and for causal prefill rows."""
+    rng = np.random.default_rng(12)
+    hkv, hq, nb = 4, 8, 6
+    kc = np.zeros((nb, 16, hkv, 128), np.uint8)
+    vc = rng.integers(0, 120, (nb, 16, hkv, 128), dtype=np.uint8)
+    ks = rng.random((nb, 16, hkv)).astype(np.float32) + 0.5
+    vs = rng.random((nb, 16, hkv)).astype(np.float32) + 0.5
+    kp, vp = fp8.pack_pools(kc, ks, vc, vs)
+    bt = np.array([[3, 1, 4, 0], [5, 2, 0, 0]], np.int32)
+    ql, cl = np.array([5, 1]), np.array([50, 20])
+    q = _bf16(rng.standard_normal((6, hq, 128)))
+    out, lse = fp8.attention(ql, cl, bt, q, kp, vp, num_q_heads=hq, num_kv_heads=hkv)
+    vd = fp8.e4m3_decode(vc) * vs[..., None].astype(np.float64)
+    rows = [(0, 0, 45 + i, i) for i in range(5)] + [(1, 0, 19, 5)]
+    for s, _, pos, t in rows:
+        idx = np.arange(pos + 1)
+        vals = vd[bt[s, idx // 16], idx % 16]          # [pos + 1, Hkv, d]
+        for h in range(hq):
+            assert np.allclose(out[t, h], vals[:, h // 2].mean(0), atol=1e-12)
+            assert np.isclose(lse[t, h], np.log(pos + 1), atol=1e-12)
