@@ -275,11 +275,15 @@ def run_reference(args):
         ins = W.mla_expand_inputs(batch, seed=args.seed)
         slots, bt, _ = W.expanded_layout(batch)
     per = []
+    # a bounded run: short warm-up samples, and timed samples that share about
+    # 150 s (at most --ref-seconds each)
+    timed_s = min(args.ref_seconds, max(1.0, 150.0 / max(args.steps, 1)))
     for i in range(args.warmup + args.steps):
+        tgt = 0.5 if i < args.warmup else timed_s
         if args.mla_expand:
-            r = cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds=args.ref_seconds)
+            r = cpu_baseline_mla_expand(batch, ins, slots, bt, target_seconds=tgt)
         else:
-            r = (cpu_baseline_fp8 if args.kv_fp8 else cpu_baseline)(batch, target_seconds=args.ref_seconds)
+            r = (cpu_baseline_fp8 if args.kv_fp8 else cpu_baseline)(batch, target_seconds=tgt)
         if i >= args.warmup:
             per.append(r)
     step_s = statistics.median(x["step_seconds_extrapolated"] for x in per)
