@@ -55,7 +55,8 @@ typedef enum {
     FNPU_EDEVICE_TIMEOUT = -4, /* a bounded device-side wait gave up, or a kernel
                                   found its shared memory misaligned and did nothing */
     FNPU_ENOMEM = -5,          /* device or host allocation failed */
-    FNPU_EDEVICE_RANGE = -6    /* a kernel met an out-of-range slot and skipped it */
+    FNPU_EDEVICE_RANGE = -6    /* a kernel met an out-of-range slot, context length or
+                                  block id and skipped it */
 } fnpu_status;
 
 typedef struct {
@@ -184,8 +185,9 @@ int fnpu_mixed_attn_run(const fnpu_plan *plan, const void *q, const void *k_cach
 int fnpu_plan_check(const fnpu_plan *plan, void *stream);
 
 /* Synchronise `stream`, then read and clear the library-wide device error
- * flag of the current device (set by fnpu_kv_append on an out-of-range slot):
- * FNPU_OK, FNPU_EDEVICE_RANGE or FNPU_ECUDA. */
+ * flag of the current device (set by fnpu_kv_append on an out-of-range slot,
+ * and by fnpu_decode_attn_noalloc on a context length or block id out of
+ * range): FNPU_OK, FNPU_EDEVICE_RANGE or FNPU_ECUDA. */
 int fnpu_check(void *stream);
 
 /* Release the plan and its device workspace. Waits for the plan's stream
@@ -251,6 +253,13 @@ int fnpu_dispatch_next_share(int32_t share_pct, float prefill_ms, float decode_m
  *   q             device bf16 [num_seqs, Hq, d]; out bf16 [num_seqs, Hq, d];
  *                 lse fp32 [num_seqs, Hq]; k_cache / v_cache as above
  * Supports split K/V caches with d_qk = d_v in {64, 128} and Hq/Hkv <= 8.
+ * The context lengths and block ids are device data, so the kernel checks
+ * them: a sequence whose context_len lies outside [1, max_context_len] is
+ * skipped (its out and lse rows are left as they were), and a block id
+ * outside [0, num_blocks) is never loaded (the sequence's result is then
+ * undefined); either raises the library-wide device error flag, which
+ * fnpu_check reports as FNPU_EDEVICE_RANGE. No load leaves the block-table
+ * rows or the pools.
  * Errors: FNPU_EINVAL for bad arguments and for requests whose scratch
  * (4 B per counter, plus 4 B * (Hq/Hkv) * (d + 1) per split, for
  * num_seqs * Hkv * ceil(max_context_len / split_keys) splits) exceeds

@@ -16,7 +16,12 @@
 //     every GPU that loads this library holds from load until the process
 //     exits; requests that need more are rejected;
 //   * the counters are cleared with cudaMemsetAsync at the start of every
-//     call (it allocates nothing).
+//     call (it allocates nothing);
+//   * the context lengths and block ids are only seen on the device, so the
+//     kernel checks them there: a context outside [1, max_context_len] is
+//     skipped, and a block id outside [0, num_blocks) is never loaded; both
+//     raise the library-wide device error flag (fnpu_check reports it), and
+//     no load leaves the caller's block-table rows or pools.
 //
 // The host code cannot pass g_noalloc_scratch itself to a kernel: in host code
 // that name is a host-side shadow, not a device address. The device address
@@ -48,6 +53,8 @@ struct NoallocParams {
     const int32_t *block_table;
     int32_t bt_stride, num_q_heads, num_kv_heads, group, block_size;
     int32_t max_splits, split_keys;
+    int32_t max_context_len, num_blocks;  // the host's bounds, checked on the device
+    int32_t *err;                         // library-wide device error flag (bit 1)
     int64_t k_slot_stride, v_slot_stride;
     float scale_log2;
     int32_t *counters;  // [num_seqs * Hkv] inside the scratch
@@ -72,9 +79,16 @@ __global__ void __launch_bounds__(kThreads, 2) decode_noalloc_kernel(const Noall
     const int kvh = grp % p.num_kv_heads;
     const int seq = grp / p.num_kv_heads;
     const int ctx = p.context_len[seq];
-    int nsp = (ctx + p.split_keys - 1) / p.split_keys;
-    if (nsp > p.max_splits) nsp = p.max_splits;  // the last split then runs to the end
-    if (split >= nsp || ctx <= 0) return;
+    if (ctx < 1 || ctx > p.max_context_len) {
+        // the host's bound sized the grid and the block-table rows: such a
+        // sequence is skipped (its out and lse rows are left as they were)
+        if (split == 0 && threadIdx.x == 0) atomicOr(p.err, 2);
+        return;
+    }
+    // ctx <= max_context_len, so nsp <= max_splits and every key's block-table
+    // entry lies inside the row (stride >= ceil(max_context_len / bs))
+    const int nsp = (ctx + p.split_keys - 1) / p.split_keys;
+    if (split >= nsp) return;
     const int key_begin = split * p.split_keys;
     const int key_end = (split == nsp - 1) ? ctx : key_begin + p.split_keys;
 
@@ -106,9 +120,19 @@ __global__ void __launch_bounds__(kThreads, 2) decode_noalloc_kernel(const Noall
         for (int i = tid; i < kTileKeys * kChunks; i += kThreads) {
             const int row = i / kChunks, ch = i % kChunks;
             const int key = kb + row;
-            const bool valid = key < key_end;
+            bool valid = key < key_end;
             int64_t slot = 0;
-            if (valid) slot = static_cast<int64_t>(__ldg(bt + key / bs)) * bs + key % bs;
+            if (valid) {
+                const int blk = __ldg(bt + key / bs);
+                if (blk < 0 || blk >= p.num_blocks) {
+                    // never loaded (the stage is zero-filled); the result of
+                    // this sequence is undefined and the flag says so
+                    valid = false;
+                    if (ch == 0) atomicOr(p.err, 2);
+                } else {
+                    slot = static_cast<int64_t>(blk) * bs + key % bs;
+                }
+            }
             const uint32_t off = swz_off(row, ch, D * 2);
             cp_async_16(sK + off, p.k_cache + slot * p.k_slot_stride + kvh * D + ch * 8, valid);
             cp_async_16(sV + off, p.v_cache + slot * p.v_slot_stride + kvh * D + ch * 8, valid);
@@ -327,6 +351,9 @@ extern "C" int fnpu_decode_attn_noalloc(const fnpu_attn_desc *desc, int32_t num_
     float *scratch = nullptr;
     int rc = scratch_address(&scratch);
     if (rc != FNPU_OK) return rc;
+    int *err = nullptr;
+    rc = global_error_address(&err);
+    if (rc != FNPU_OK) return rc;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaMemsetAsync(scratch, 0, sizeof(int32_t) * static_cast<size_t>(groups), st) != cudaSuccess)
         return FNPU_ECUDA;
@@ -346,6 +373,9 @@ extern "C" int fnpu_decode_attn_noalloc(const fnpu_attn_desc *desc, int32_t num_
     p.block_size = desc->block_size;
     p.max_splits = static_cast<int32_t>(max_splits);
     p.split_keys = split_keys;
+    p.max_context_len = max_context_len;
+    p.num_blocks = desc->num_blocks;
+    p.err = err;
     p.k_slot_stride = static_cast<int64_t>(Hkv) * D;
     p.v_slot_stride = static_cast<int64_t>(Hkv) * D;
     const float scale = desc->softmax_scale > 0.f ? desc->softmax_scale

@@ -125,6 +125,9 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
                      const int64_t *slots, int32_t num_tokens, void *k_cache, void *v_cache,
                      void *stream);
 int read_and_clear_global_error(void *stream, int *flag);
+// Device address of the library-wide error flag on the current device (looked
+// up once per device), for kernels of other translation units that raise it.
+int global_error_address(int **out);
 // MLA expansion: gather the c parts of latent rows (512 + 64 columns) into ws
 // [n, 512] and broadcast their r parts into columns 128..191 of k_out [n, heads, 192]
 int launch_mla_gather(const void *latent, const int64_t *slots, int32_t n, int64_t num_slots, int32_t heads,

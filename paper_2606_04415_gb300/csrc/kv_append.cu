@@ -8,12 +8,16 @@
 // bit-exact.
 #include <cuda_fp8.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace fnpu {
 
-// Library-wide device error flag (bit 0: out-of-range slot), one per device
-// that loads the library; read and cleared by fnpu_check().
+// Library-wide device error flag, one per device that loads the library;
+// read and cleared by fnpu_check(). Bit 0: an append met an out-of-range
+// slot; bit 1: the allocation-free decode met a context length or a block
+// id out of range.
 __device__ int g_device_error = 0;
 
 __global__ void __launch_bounds__(256) kv_append_kernel(
@@ -203,6 +207,26 @@ int launch_mla_gather(const void *latent, const int64_t *slots, int32_t n, int64
         static_cast<const uint4 *>(latent), slots, n, num_slots, heads, static_cast<uint4 *>(ws),
         static_cast<uint4 *>(k_out));
     return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
+}
+
+int global_error_address(int **out) {
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static int *addr[kMaxDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return FNPU_ECUDA;
+    if (dev < 0 || dev >= kMaxDevices) return FNPU_EUNSUPPORTED;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!addr[dev]) {
+        void *ptr = nullptr;
+        if (cudaGetSymbolAddress(&ptr, g_device_error) != cudaSuccess || !ptr) {
+            cudaGetLastError();
+            return FNPU_ECUDA;
+        }
+        addr[dev] = static_cast<int *>(ptr);
+    }
+    *out = addr[dev];
+    return FNPU_OK;
 }
 
 int read_and_clear_global_error(void *stream, int *flag) {
