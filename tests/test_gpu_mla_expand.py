@@ -10,11 +10,20 @@ of a rounding boundary (about 1% of them, asserted below).
 
 Attention kernel alone (random 192-wide keys and 128-wide values from the
 seeded generator): |O - O_ref| <= 2e-2, |LSE - LSE_ref| <= 1e-3 as for every
-attention path. End to end (expansion then attention), the reference runs on
-its own expanded rows; a key element one bf16 unit off moves a score by up to
-scale * |q_d| * 2^-7 |k_d| (about 5e-4 for N(0, 1) data at the tails), and a
-few such elements in a row move the log-sum-exp by up to about 2e-3: the LSE
-bound there is 3e-3 (O stays 2e-2).
+attention path.
+
+End to end (expansion then attention) the reference attends over its own
+expanded rows K_r, V_r and the GPU over K_g, V_g, so the kernel tolerances
+hold against attention over K_g, V_g, and the distance between the two
+attentions is bounded from the measured differences, per (token, head), with
+no fixed constant:
+  * score j moves by |<q, K_g,j - K_r,j>| * scale <= ds_j =
+    scale * sum_d |q_d| |K_g - K_r|_jd;
+  * the log-sum-exp is 1-Lipschitz in the max norm of the scores, so
+    |LSE_g - LSE_r| <= 1e-3 + max_j ds_j over the visible keys;
+  * with D = max_j ds_j every softmax weight moves by a factor within
+    [e^-2D, e^2D], so sum_j |w_g,j - w_r,j| <= e^2D - 1, and per column
+    |O_g - O_r| <= 2e-2 + max_j |V_g - V_r|_j + (e^2D - 1) max_j |V_r|_j.
 """
 import numpy as np
 import pytest
@@ -28,7 +37,6 @@ pytestmark = pytest.mark.gpu
 
 O_TOL = 2e-2
 LSE_TOL = 1e-3
-LSE_TOL_EXPANDED = 3e-3  # end to end: flipped bf16 roundings of the expanded keys (see above)
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -37,6 +45,42 @@ def _cuda():
         pytest.skip("no CUDA device")
     import paper_2606_04415_gb300 as fnpu
     fnpu.load()
+
+
+def _expansion_bounds(batch, bt, q_bits, gk, gv, kb, vb, toks):
+    """Per checked (token, head): the bound on |LSE_g - LSE_r| and, per column,
+    on |O_g - O_r| that the expansion differences allow (module docstring).
+    Expanded rows of sequence s are bt[s, 0] * 16 + position."""
+    H = gk.shape[1]
+    qs = batch.query_start
+    seq_of = np.searchsorted(qs, toks, side="right") - 1
+    pos = (batch.context_len[seq_of] - batch.query_len[seq_of] + (toks - qs[seq_of])).astype(np.int64)
+    first = bt[seq_of, 0].astype(np.int64) * 16
+    scale = 1.0 / np.sqrt(192.0)
+    qabs = np.abs(X.bf16_bits_to_f64(q_bits[toks]))          # [t, H, 192]
+    dk = np.abs(X.bf16_bits_to_f64(gk) - X.bf16_bits_to_f64(kb))  # [n, H, 192]
+    dv = np.abs(X.bf16_bits_to_f64(gv) - X.bf16_bits_to_f64(vb))  # [n, H, 128]
+    va = np.abs(X.bf16_bits_to_f64(vb))
+    n = dk.shape[0]
+    rows = np.arange(n)
+    vis = (rows[None, :] >= first[:, None]) & (rows[None, :] <= (first + pos)[:, None])
+    dmax = np.empty((len(toks), H))
+    for h in range(H):
+        ds = scale * (qabs[:, h, :] @ dk[:, h, :].T)          # [t, n]
+        dmax[:, h] = np.where(vis, ds, 0.0).max(axis=1)
+    # maxima over the visible rows j <= pos: running maxima along each sequence
+    dv_vis = np.empty((len(toks), H, 128))
+    va_vis = np.empty((len(toks), H, 128))
+    for s in np.unique(seq_of):
+        r0, c = int(bt[s, 0]) * 16, int(batch.context_len[s])
+        cdv = np.maximum.accumulate(dv[r0:r0 + c], axis=0)
+        cva = np.maximum.accumulate(va[r0:r0 + c], axis=0)
+        sel = seq_of == s
+        dv_vis[sel] = cdv[pos[sel]]
+        va_vis[sel] = cva[pos[sel]]
+    lse_bound = LSE_TOL + dmax
+    o_bound = O_TOL + dv_vis + np.expm1(2.0 * dmax)[:, :, None] * va_vis
+    return lse_bound, o_bound
 
 
 def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
@@ -68,12 +112,13 @@ def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
     ref_o, ref_l = oracle.attention(batch.query_len, batch.context_len, bt, ins["q"], kb, vb, num_q_heads=heads,
                                     num_kv_heads=heads, head_dim_qk=192, head_dim_v=128, block_size=16,
                                     tokens=tokens)
-    if tokens is not None:
-        out, lse = out[tokens], lse[tokens]
+    toks = np.arange(batch.num_tokens, dtype=np.int64) if tokens is None else np.asarray(tokens, np.int64)
+    out, lse = out[toks], lse[toks]
     assert np.isfinite(out).all() and np.isfinite(lse).all()
-    eo, el = np.abs(out - ref_o).max(), np.abs(lse - ref_l).max()
-    assert eo <= O_TOL, f"max |dO| = {eo}"
-    assert el <= LSE_TOL_EXPANDED, f"max |dLSE| = {el}"
+    lse_bound, o_bound = _expansion_bounds(batch, bt, ins["q"], gk, gv, kb, vb, toks)
+    dl, do = np.abs(lse - ref_l), np.abs(out - ref_o)
+    assert np.all(dl <= lse_bound), f"max |dLSE| - bound = {float(np.max(dl - lse_bound))}"
+    assert np.all(do <= o_bound), f"max |dO| - bound = {float(np.max(do - o_bound))}"
     return st
 
 
