@@ -420,7 +420,7 @@ def run_fnpu_mla_expand(args):
     F_gemm = 2.0 * n * 512 * 128 * H * 2
     F_attn = 2.0 * H * W.pairs(batch) * (192 + 128)
     roof = {"bound": "tensor", "achieved": F_attn / (t_att * 1e-3) / 1e12, "peak": peaks["bf16_tflops"],
-            "unit": "TFLOP/s", "kernel": "prefill_mma_kernel<192, 128> (the attention call)"}
+            "unit": "TFLOP/s", "kernel": "prefill_tc_kernel<192, 128> (the attention call)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["traffic"] = args.traffic
     roof["peak_source"] = peaks["source"] + " burst"
@@ -438,7 +438,7 @@ def run_fnpu_mla_expand(args):
         "kernel_ms": {"append": t_app, "expand": t_exp, "attention": t_att},
         "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
-        "gpu_launches": K * 3,  # append, gather, attention (plus two cuBLAS GEMM launches per step)
+        "gpu_launches": K * (3 + st.plan.info()["launches_per_run"]),  # append, gather, GEMM, attention
         "clocks": clk,
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -483,16 +483,23 @@ def run_fnpu(args):
         st = DeviceStep(batch, opts=opts, device=str(dev), kv_fp8=True, pool_init=init)
     else:
         st = DeviceStep(batch, opts=opts, device=str(dev))
-    # the plan (host: validation, work lists, workspace, one async upload),
-    # timed apart from the step: median host time of a few plans of the batch
+    # the plan (host: validation, work lists, one async upload), timed apart
+    # from the step: median host time of re-plans of the batch into one plan
+    # (the steady state of a serving loop, which plans every step), and of
+    # new plans (which also allocate the workspace, staging, streams, events)
     torch.cuda.synchronize(dev)
-    plan_ms = []
+    planner_ms, first_ms = [], []
+    extra = None
     for _ in range(5):
         t0 = time.perf_counter()
         extra = fnpu.mixed_attn_plan(st.desc, batch.query_len, batch.context_len, batch.phase, batch.block_table,
                                      opts=opts)
-        plan_ms.append((time.perf_counter() - t0) * 1e3)
+        first_ms.append((time.perf_counter() - t0) * 1e3)
         extra.destroy()
+    for _ in range(20):
+        t0 = time.perf_counter()
+        st.replan(opts)
+        planner_ms.append((time.perf_counter() - t0) * 1e3)
     torch.cuda.synchronize(dev)
     info = st.plan.info()
     stream = torch.cuda.current_stream(dev)
@@ -522,6 +529,16 @@ def run_fnpu(args):
     torch.cuda.synchronize(dev)
     if fnpu.plan_check(st.plan) != fnpu.FNPU_OK or fnpu.check() != fnpu.FNPU_OK:
         raise RuntimeError("device error flag raised during warm-up")
+    # re-plans at the decode share the dispatch settled on: what a serving loop
+    # pays every step once its controller has converged
+    share_opts = fnpu.PlanOpts(args.split, share if args.dispatch == "feedback" else args.decode_share, 0,
+                               args.flags)
+    plan_ms = []
+    for _ in range(20):
+        t0 = time.perf_counter()
+        st.replan(share_opts)
+        plan_ms.append((time.perf_counter() - t0) * 1e3)
+    torch.cuda.synchronize(dev)
 
     K = args.steps
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
@@ -556,25 +573,37 @@ def run_fnpu(args):
     h_l = torch.empty(st.lse.shape, dtype=torch.float32).pin_memory()
     h2d = sum(x.numel() * x.element_size() for x in (h_q, h_k, h_v, h_s) if x is not None)
     d2h = h_o.numel() * h_o.element_size() + h_l.numel() * h_l.element_size()
-    e2e_ms = []
-    for i in range(args.warmup + K):
-        _flush_l2(flush, flush_r)
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        st.q.copy_(h_q, non_blocking=True)
-        st.k_new.copy_(h_k, non_blocking=True)
-        if h_v is not None:
-            st.v_new.copy_(h_v, non_blocking=True)
-        st.slot_mapping.copy_(h_s, non_blocking=True)
-        st.run()
-        h_o.copy_(st.out, non_blocking=True)
-        h_l.copy_(st.lse, non_blocking=True)
-        b.record(stream)
-        b.synchronize()
-        if i >= args.warmup:
-            e2e_ms.append(a.elapsed_time(b))
-    e2e = max_over_ranks(sum(e2e_ms) / len(e2e_ms), ws, dev)
+    # (a second pass re-plans the step from its host metadata every step, as a
+    # serving loop whose metadata changes does: the device is idle when the
+    # timed region starts, so the plan's host time, the enqueueing and the
+    # metadata upload all lie inside it)
+    e2e_by_mode = {}
+    for mode in ("plan_once", "replan_every_step"):
+        e2e_ms = []
+        for i in range(args.warmup + K):
+            _flush_l2(flush, flush_r)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            if mode == "replan_every_step":
+                torch.cuda.synchronize(dev)
+            a.record(stream)
+            if mode == "replan_every_step":
+                st.replan(share_opts)
+            st.q.copy_(h_q, non_blocking=True)
+            st.k_new.copy_(h_k, non_blocking=True)
+            if h_v is not None:
+                st.v_new.copy_(h_v, non_blocking=True)
+            st.slot_mapping.copy_(h_s, non_blocking=True)
+            st.run()
+            h_o.copy_(st.out, non_blocking=True)
+            h_l.copy_(st.lse, non_blocking=True)
+            b.record(stream)
+            b.synchronize()
+            if i >= args.warmup:
+                e2e_ms.append(a.elapsed_time(b))
+        e2e_by_mode[mode] = max_over_ranks(sum(e2e_ms) / len(e2e_ms), ws, dev)
+    e2e = e2e_by_mode["plan_once"]
+    e2e_replan = e2e_by_mode["replan_every_step"]
 
     # roofline of the dominant kernel work (the attention launch): algorithmic
     # FLOPs and bytes per run / measured duration
@@ -604,7 +633,9 @@ def run_fnpu(args):
         "config": {"workload": args.workload, "seed": args.seed, "query_tokens": T,
                    "num_seqs": batch.num_seqs, "prefill_ctx": int(batch.context_len[0]),
                    "flops": F, "bytes": work["bytes"], "l2": "flushed between timed steps (512 MB write, then 256 MB read)",
-                   "plan": info, "plan_host_ms": round(statistics.median(plan_ms), 3),
+                   "plan": info, "plan_host_ms": round(statistics.median(plan_ms), 4),
+                   "plan_host_ms_planner_share": round(statistics.median(planner_ms), 4),
+                   "plan_host_ms_new_plan": round(statistics.median(first_ms), 3),
                    "dispatch": args.dispatch, "kv_cache": "fp8_e4m3" if args.kv_fp8 else "bf16"},
         "roofline": roof,
         "roofline_step_frac": {"burst": step_roof / (step_ms * 1e-3),
@@ -612,7 +643,8 @@ def run_fnpu(args):
                                "denominator": "max(F/bf16 peak, B/HBM peak) of measured"},
         "kernel_ms": {"append": sum(t_append) / K, "attention": attn_ms},
         "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e,
+                "replan_every_step": {"value": job_throughput(ws, T, e2e_replan), "ms_per_step": e2e_replan}},
         "gpu_launches": K * (1 + info["launches_per_run"]),
         "clocks": clk,
     }

@@ -168,6 +168,29 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs,
                             void *stream, fnpu_plan **out);
 
 /*
+ * Re-plan: rebuild `plan` for a new step's metadata (same descriptor; the
+ * arguments as for fnpu_mixed_attn_plan_ex), keeping what the plan already
+ * holds -- its streams, events and green contexts, two pinned staging
+ * buffers used in turn, and its device workspace, which is reallocated only
+ * when the new step needs more than it holds (then with a quarter of
+ * headroom, after waiting for the device). In a serving loop whose metadata
+ * changes every step (the phase-aware dispatch of Sec. 3.4 plans every step
+ * anew) this makes the plan host work alone: no allocation, stream or event
+ * creation in the steady state. Green contexts are rebuilt only when the
+ * decode share asks for a different partition.
+ * The metadata upload is enqueued on `stream`. Runs of the plan already
+ * enqueued on `stream` finish before it; runs enqueued on other streams must
+ * be ordered before this call's upload by the caller. The plan's error flag
+ * is kept (fnpu_plan_check still reports a failed earlier run).
+ * Errors: as fnpu_mixed_attn_plan_ex; on FNPU_EINVAL or FNPU_EUNSUPPORTED
+ * from the argument checks the plan is unchanged; after any other error it
+ * must be re-planned successfully or destroyed before it runs again.
+ */
+int fnpu_mixed_attn_replan(fnpu_plan *plan, int32_t num_seqs, const int32_t *query_len,
+                           const int32_t *context_len, const uint8_t *phase, const int32_t *block_table,
+                           int32_t block_table_stride, const fnpu_plan_opts *opts, void *stream);
+
+/*
  * Attention for every query of the planned step. q, k_cache, v_cache, out,
  * lse are device pointers in the layouts above (v_cache NULL for latent;
  * with kv_fp8 = 1, k_cache and v_cache are the FP8 byte pools).
@@ -311,13 +334,17 @@ int fnpu_version(void);
  *   w_uk, w_uv    device bf16 [Hq, 512, 128] (row-major per head)
  *   workspace     device, at least n * 512 * 2 bytes (scratch; caller-owned)
  *   k_out         device bf16 [n, Hq, 192];  v_out device bf16 [n, Hq, 128]
- * The two products are cuBLAS strided-batched GEMMs on the stream (one
- * batch entry per head); the gather is this library's kernel.
+ * Two kernels of this library on the stream: a gather of the c parts into
+ * the workspace (and of the r parts into every head's key), then one
+ * tcgen05 GEMM (per CTA 256 rows x one head's 128 key and 128 value
+ * columns, fp32 accumulators in tensor memory) for both products.
  * Errors: FNPU_EINVAL for NULL or misaligned pointers (16 bytes; slots 8),
  * n < 0 or a desc that is not a latent cache; FNPU_EUNSUPPORTED for other
- * latent widths; FNPU_ECUDA if a CUDA or cuBLAS call fails. A slot >=
+ * latent widths; FNPU_ECUDA if a CUDA call fails. A slot >=
  * num_blocks * block_size gives a zero row and raises the device error
- * flag (FNPU_EDEVICE_RANGE from fnpu_check).
+ * flag (FNPU_EDEVICE_RANGE from fnpu_check); a bounded wait of the GEMM
+ * that gives up leaves its rows undefined and makes fnpu_check return
+ * FNPU_EDEVICE_TIMEOUT.
  */
 int fnpu_mla_expand(const fnpu_attn_desc *desc, const void *latent_cache, const int64_t *slots, int32_t n,
                     const void *w_uk, const void *w_uv, void *workspace, void *k_out, void *v_out,

@@ -6,6 +6,7 @@ kernels. Functions carry the C names without the ``fnpu_`` prefix:
 
     kv_append(desc, k_new, v_new, slot_mapping, k_cache, v_cache, stream=None)
     mixed_attn_plan(desc, query_len, context_len, phase, block_table, opts=None, stream=None)
+    mixed_attn_replan(plan, query_len, context_len, phase, block_table, opts=None, stream=None)
     mixed_attn_run(plan, q, k_cache, v_cache, out, lse, stream=None)
     check(stream=None), plan_check(plan, stream=None), status_str(code)
 
@@ -40,7 +41,7 @@ EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
     "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error", "fnpu_plan_phase_ms",
-    "fnpu_dispatch_next_share", "fnpu_mla_expand",
+    "fnpu_dispatch_next_share", "fnpu_mla_expand", "fnpu_mixed_attn_replan",
 )
 
 
@@ -89,6 +90,7 @@ def load(build_if_missing: bool = True):
                                          ctypes.POINTER(P)]
     lib.fnpu_mixed_attn_plan_ex.argtypes = [ctypes.POINTER(AttnDesc), i32, P, P, P, P, i32,
                                             ctypes.POINTER(PlanOpts), P, ctypes.POINTER(P)]
+    lib.fnpu_mixed_attn_replan.argtypes = [P, i32, P, P, P, P, i32, ctypes.POINTER(PlanOpts), P]
     lib.fnpu_mixed_attn_run.argtypes = [P, P, P, P, P, P, P]
     lib.fnpu_mla_expand.argtypes = [ctypes.POINTER(AttnDesc), P, P, i32, P, P, P, P, P, P]
     lib.fnpu_plan_check.argtypes = [P, P]
@@ -109,7 +111,7 @@ def load(build_if_missing: bool = True):
     for name in ("fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex",
                  "fnpu_mixed_attn_run", "fnpu_plan_check", "fnpu_check", "fnpu_plan_info",
                  "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_plan_phase_ms",
-                 "fnpu_dispatch_next_share", "fnpu_mla_expand"):
+                 "fnpu_dispatch_next_share", "fnpu_mla_expand", "fnpu_mixed_attn_replan"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -232,6 +234,24 @@ def mixed_attn_plan(desc: AttnDesc, query_len, context_len, phase, block_table,
     if rc != FNPU_OK:
         raise FnpuError(rc, "fnpu_mixed_attn_plan")
     return Plan(out.value, desc, int(ql.sum()))
+
+
+def mixed_attn_replan(plan: Plan, query_len, context_len, phase, block_table,
+                      opts: Optional[PlanOpts] = None, stream=None) -> None:
+    """Rebuild ``plan`` for a new step's metadata, reusing its streams, events,
+    staging and workspace (``fnpu_mixed_attn_replan``)."""
+    ql = _np(query_len, np.int32)
+    cl = _np(context_len, np.int32)
+    ph = _np(phase, np.uint8)
+    bt = _np(block_table, np.int32)
+    if bt.ndim != 2 or not (ql.shape == cl.shape == ph.shape) or bt.shape[0] != ql.shape[0]:
+        raise ValueError("metadata shapes disagree")
+    rc = load().fnpu_mixed_attn_replan(plan.handle, int(ql.shape[0]), ql.ctypes.data, cl.ctypes.data,
+                                       ph.ctypes.data, bt.ctypes.data, int(bt.shape[1]),
+                                       None if opts is None else ctypes.byref(opts), _stream(stream))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_mixed_attn_replan")
+    plan.num_tokens = int(ql.sum())
 
 
 def mixed_attn_run(plan: Plan, q, k_cache, v_cache, out, lse, stream=None) -> None:

@@ -72,8 +72,7 @@ def build(force: bool = False, verbose: bool = False, ptxas_verbose: bool = Fals
     with cf.ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as ex:
         objs = list(ex.map(compile_one, srcs))
     tmp = LIB + f".tmp{os.getpid()}"
-    # cuBLAS: the two plain GEMMs of the MLA expansion (fnpu_mla_expand)
-    r = subprocess.run([nvcc, *ARCH, "-shared", "-o", tmp, *objs, "-lcublas"], capture_output=True, text=True)
+    r = subprocess.run([nvcc, *ARCH, "-shared", "-o", tmp, *objs], capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
     os.replace(tmp, LIB)

@@ -40,9 +40,17 @@ struct fnpu_plan {
     int32_t num_mgroups = 0;  // split decode tokens merged by the merge kernel
     fnpu::MergeGroup *d_mgroups = nullptr;  // decode on the TMA-fed persistent kernel (items cover all kv heads)
     int32_t num_ditems = 0, num_pitems = 0, num_groups = 0, num_parts = 0;
+    // device workspace: the error flag and work queues at offset 0 (kept
+    // across re-plans), then metadata and scratch; it grows only when a
+    // re-plan needs more than ws_cap bytes
     void *d_ws = nullptr;
-    size_t ws_bytes = 0;
-    void *h_stage = nullptr;
+    size_t ws_bytes = 0, ws_cap = 0;
+    // pinned staging of the metadata upload, two buffers used in turn; the
+    // event after each upload says when its buffer may be rewritten
+    void *h_stage[2] = {nullptr, nullptr};
+    size_t stage_cap[2] = {0, 0};
+    cudaEvent_t e_upload[2] = {nullptr, nullptr};
+    int32_t stage_turn = 0;
     fnpu::SeqInfo *d_seqs = nullptr;
     int32_t *d_bt = nullptr;
     fnpu::DecodeItem *d_ditems = nullptr;
@@ -73,6 +81,8 @@ struct fnpu_plan {
     // disjoint SM partitions (dec_sms SMs for decode, pre_ctas for prefill)
     CUgreenCtx g_pre = nullptr, g_dec = nullptr;
     int32_t dec_sms = 0;
+    int32_t green_k = -1;  // decode SMs asked of the current green contexts
+    int32_t green_pre = 0;  // SMs of their prefill partition
 };
 
 namespace fnpu {
@@ -123,18 +133,39 @@ const GreenApi &green_api() {
     return g;
 }
 
-void destroy_sync_objects(fnpu_plan *pl) {
+// The co-location streams (and green contexts) of a plan.
+void destroy_streams(fnpu_plan *pl) {
     if (pl->s_pre) cudaStreamDestroy(pl->s_pre);
     if (pl->s_dec) cudaStreamDestroy(pl->s_dec);
     if (pl->g_pre) green_api().destroy(pl->g_pre);
     if (pl->g_dec) green_api().destroy(pl->g_dec);
     pl->g_pre = pl->g_dec = nullptr;
+    pl->s_pre = pl->s_dec = nullptr;
+    pl->green_k = -1;
+}
+
+void destroy_sync_objects(fnpu_plan *pl) {
+    destroy_streams(pl);
     if (pl->e_started) cudaEventDestroy(pl->e_started);
     if (pl->e_dec) cudaEventDestroy(pl->e_dec);
     if (pl->e_fork) cudaEventDestroy(pl->e_fork);
     if (pl->e_pre) cudaEventDestroy(pl->e_pre);
-    pl->s_pre = pl->s_dec = nullptr;
     pl->e_fork = pl->e_started = pl->e_pre = pl->e_dec = nullptr;
+}
+
+// Everything a plan owns; the plan itself is deleted by the caller.
+void release_plan(fnpu_plan *pl) {
+    destroy_sync_objects(pl);
+    for (int i = 0; i < 2; ++i) {
+        if (pl->e_upload[i]) cudaEventDestroy(pl->e_upload[i]);
+        if (pl->h_stage[i]) cudaFreeHost(pl->h_stage[i]);
+        pl->e_upload[i] = nullptr;
+        pl->h_stage[i] = nullptr;
+        pl->stage_cap[i] = 0;
+    }
+    if (pl->d_ws) cudaFree(pl->d_ws);
+    pl->d_ws = nullptr;
+    pl->ws_cap = 0;
 }
 
 // Modelled rates of the two phases (measured on the co-located Qwen2.5-7B
@@ -145,7 +176,9 @@ constexpr double kTileSec = 1.5e-6;
 constexpr double kDecodeSmBps = 69e9;
 constexpr double kDecodeAllBps = 4.0e12;
 
-int64_t lpt_makespan(const std::vector<int64_t> &costs, int32_t m);
+// (stop_at: the run may end as soon as the makespan reaches it)
+int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_at = INT64_MAX);
+std::vector<int32_t> cost_histogram(const std::vector<int64_t> &costs);
 
 // SMs that start on decode while the others run prefill: the prefill CTAs on
 // sms - k SMs take the items longest first, so they last about the LPT
@@ -158,8 +191,9 @@ int32_t choose_decode_sms(const std::vector<int64_t> &item_tiles, double tile_sc
                           int32_t sms) {
     int32_t best_k = 1;
     double best_t = -1.0;
+    const std::vector<int32_t> hist = cost_histogram(item_tiles);
     for (int32_t k = 1; k <= sms / 2; ++k) {
-        const double tp = static_cast<double>(lpt_makespan(item_tiles, sms - k)) * tile_scale * kTileSec;
+        const double tp = static_cast<double>(lpt_makespan(hist, sms - k)) * tile_scale * kTileSec;
         const double rate = std::min(kDecodeAllBps, k * kDecodeSmBps);
         const double left = std::max(0.0, static_cast<double>(dec_bytes) - tp * rate);
         const double t = tp + left / kDecodeAllBps;
@@ -190,17 +224,52 @@ int32_t split_bound(int32_t ntiles, int32_t n, int32_t j) {
     return static_cast<int32_t>((static_cast<int64_t>(ntiles) * j) / n);
 }
 
-// Longest-processing-time-first makespan of `costs` (sorted descending) on m
-// workers.
-int64_t lpt_makespan(const std::vector<int64_t> &costs, int32_t m) {
-    std::vector<int64_t> heap(static_cast<size_t>(std::max(m, 1)), 0);  // min-heap of loads
-    auto cmp = [](int64_t a, int64_t b) { return a > b; };
-    for (int64_t c : costs) {
-        std::pop_heap(heap.begin(), heap.end(), cmp);
-        heap.back() += c;
-        std::push_heap(heap.begin(), heap.end(), cmp);
+// Item costs (positive integers, in tiles) as a histogram: hist[c] items of
+// cost c.
+std::vector<int32_t> cost_histogram(const std::vector<int64_t> &costs) {
+    int64_t cmax = 0;
+    for (int64_t c : costs) cmax = std::max(cmax, c);
+    std::vector<int32_t> hist(static_cast<size_t>(cmax) + 1, 0);
+    for (int64_t c : costs) ++hist[static_cast<size_t>(std::max<int64_t>(c, 0))];
+    return hist;
+}
+
+// Longest-processing-time-first makespan of the items of `hist` on m workers:
+// the items longest first, each to the least loaded worker. The loads are
+// integers and the least load never decreases (the worker that takes an item
+// had the least load), so a count of workers per load value with a pointer
+// that only moves up finds the least loaded workers; the items of one cost go
+// to them together (workers are interchangeable, so the loads evolve as with
+// one item at a time). No load exceeds the mean plus the largest item, which
+// bounds the counts. Linear in distinct costs + loads.
+int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_at) {
+    m = std::max<int32_t>(m, 1);
+    int64_t total = 0, n = 0;
+    for (size_t c = 0; c < hist.size(); ++c) {
+        total += static_cast<int64_t>(c) * hist[c];
+        n += hist[c];
     }
-    return *std::max_element(heap.begin(), heap.end());
+    if (n == 0) return 0;
+    const int64_t cmax = static_cast<int64_t>(hist.size()) - 1;
+    const size_t bound = static_cast<size_t>(total / m + cmax + 1);
+    thread_local std::vector<int32_t> cnt;
+    cnt.assign(bound + 1, 0);
+    cnt[0] = m;
+    size_t p = 0;
+    int64_t span = 0;
+    for (int64_t c = cmax; c >= 0; --c) {
+        int64_t k = hist[static_cast<size_t>(c)];
+        while (k > 0) {
+            while (cnt[p] == 0) ++p;
+            const int64_t t = std::min<int64_t>(cnt[p], k);
+            cnt[p] -= static_cast<int32_t>(t);
+            cnt[p + static_cast<size_t>(c)] += static_cast<int32_t>(t);
+            span = std::max<int64_t>(span, static_cast<int64_t>(p) + c);
+            k -= t;
+            if (span >= stop_at) return span;  // the caller only wants spans below stop_at
+        }
+    }
+    return span;
 }
 
 // Number of key splits per unit. A persistent CTA per SM takes items longest
@@ -220,21 +289,46 @@ std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int
     for (int j = 1; j <= 8; ++j) caps.push_back((total + static_cast<int64_t>(sms) * j - 1) / (static_cast<int64_t>(sms) * j));
     std::vector<int32_t> best(units.size(), 1), ns(units.size(), 1);
     int64_t best_span = -1;
-    std::vector<int64_t> costs;
+    {  // drop repeated candidates, keeping the first of each (ties go to the earlier one)
+        std::vector<int64_t> uniq;
+        for (int64_t c : caps)
+            if (std::find(uniq.begin(), uniq.end(), c) == uniq.end()) uniq.push_back(c);
+        caps.swap(uniq);
+    }
+    std::vector<int32_t> hist(static_cast<size_t>(maxc + kTcItemCost + kTcMergeCost) + 1);
+    // the most splits a unit can take (at most 16): its last split must start
+    // at or before max_start, and that start, floor(ntiles (n - 1) / n), does
+    // not decrease with n, so the feasible counts are 1 .. nmax
+    std::vector<int32_t> nmax(units.size(), 1);
+    for (size_t i = 0; i < units.size(); ++i) {
+        int32_t n = 16;
+        while (n > 1 && split_bound(units[i].ntiles, n, n - 1) > units[i].max_start) --n;
+        nmax[i] = n;
+    }
+    std::vector<int32_t> prev;
     for (int64_t cap : caps) {
         if (cap < 4) continue;
-        costs.clear();
+        // ceil(ntiles / cap) = floor((ntiles - 1) / cap) + 1 in double, exact
+        // for tile counts (below 2^26): a quotient that is not an integer has a
+        // fraction of at least 1 / cap, above 1e-8, and the product errs by far
+        // less than the 1e-9 added (the conversion truncates, = floor here)
+        const double inv = 1.0 / static_cast<double>(cap);
         for (size_t i = 0; i < units.size(); ++i) {
-            const TcUnit &u = units[i];
-            int32_t n = static_cast<int32_t>(std::min<int64_t>((u.ntiles + cap - 1) / cap, 16));
-            while (n > 1 && split_bound(u.ntiles, n, n - 1) > u.max_start) --n;
-            ns[i] = n;
-            for (int32_t j = 0; j < n; ++j)
-                costs.push_back(split_bound(u.ntiles, n, j + 1) - split_bound(u.ntiles, n, j) + kTcItemCost +
-                                (n > 1 ? kTcMergeCost : 0));
+            const int32_t q = static_cast<int32_t>((units[i].ntiles - 1) * inv + 1e-9) + 1;
+            ns[i] = std::min(q, nmax[i]);
         }
-        std::sort(costs.begin(), costs.end(), [](int64_t a, int64_t b) { return a > b; });
-        const int64_t span = lpt_makespan(costs, sms);
+        if (ns == prev) continue;  // the same splits as the candidate before
+        prev = ns;
+        std::fill(hist.begin(), hist.end(), 0);
+        for (size_t i = 0; i < units.size(); ++i) {
+            // n pieces of floor(ntiles / n) or one more tiles (split_bound
+            // rounds down), the longer ones ntiles mod n of them
+            const int32_t n = ns[i], nt = units[i].ntiles, q = nt / n, r = nt % n;
+            const int32_t extra = kTcItemCost + (n > 1 ? kTcMergeCost : 0);
+            hist[static_cast<size_t>(q + 1 + extra)] += r;
+            hist[static_cast<size_t>(q + extra)] += n - r;
+        }
+        const int64_t span = lpt_makespan(hist, sms, best_span < 0 ? INT64_MAX : best_span);
         if (best_span < 0 || span < best_span) {
             best_span = span;
             best = ns;
@@ -373,6 +467,7 @@ int fnpu_check(void *stream) {
     int flag = 0;
     const int rc = read_and_clear_global_error(stream, &flag);
     if (rc != FNPU_OK) return rc;
+    if (flag & 4) return FNPU_EDEVICE_TIMEOUT;  // a bounded wait of the MLA expansion gave up
     return flag ? FNPU_EDEVICE_RANGE : FNPU_OK;
 }
 
@@ -384,60 +479,84 @@ int fnpu_mixed_attn_plan(const fnpu_attn_desc *desc, int32_t num_seqs, const int
                                    block_table_stride, nullptr, stream, out);
 }
 
-int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const int32_t *query_len,
-                            const int32_t *context_len, const uint8_t *phase,
-                            const int32_t *block_table, int32_t block_table_stride,
-                            const fnpu_plan_opts *opts, void *stream, fnpu_plan **out) {
-    int st;
-    if (!out) return FNPU_EINVAL;
-    if (!shape_ok(desc, &st)) return st;
-    if (num_seqs < 0) return FNPU_EINVAL;
-    if (num_seqs > 0 && (!query_len || !context_len || !phase || !block_table)) return FNPU_EINVAL;
-    fnpu_plan_opts o = {};
-    if (opts) o = *opts;
-    if (o.decode_split_keys < 0 || o.decode_share_pct < 0 || o.decode_share_pct > 100 || o.num_sms < 0)
-        return FNPU_EINVAL;
-    const int32_t bs = desc->block_size;
+}  // extern "C"
 
-    // validate the per-sequence metadata
+namespace {
+
+// Validated shape of one step's metadata.
+struct StepMeta {
     int64_t T = 0;
     int32_t width = 1;
     bool has_decode = false, has_prefill = false;
+};
+
+// Host checks of a plan's arguments: nothing is launched or allocated.
+int validate_meta(const fnpu_attn_desc *desc, int32_t num_seqs, const int32_t *query_len,
+                  const int32_t *context_len, const uint8_t *phase, const int32_t *block_table,
+                  int32_t block_table_stride, const fnpu_plan_opts &o, StepMeta *m) {
+    int st;
+    if (!shape_ok(desc, &st)) return st;
+    if (num_seqs < 0) return FNPU_EINVAL;
+    if (num_seqs > 0 && (!query_len || !context_len || !phase || !block_table)) return FNPU_EINVAL;
+    if (o.decode_split_keys < 0 || o.decode_share_pct < 0 || o.decode_share_pct > 100 || o.num_sms < 0)
+        return FNPU_EINVAL;
+    const int32_t bs = desc->block_size;
+    StepMeta r;
     for (int32_t s = 0; s < num_seqs; ++s) {
         const int32_t q = query_len[s], c = context_len[s];
         if (q < 1 || c < q) return FNPU_EINVAL;
         if (phase[s] > 1) return FNPU_EINVAL;
         // a decode step of several tokens (speculative verification) is causal
         // attention of a short chunk: its rows take the prefill path
-        has_decode |= phase[s] == 1 && q == 1;
-        has_prefill |= phase[s] == 0 || q > 1;
+        r.has_decode |= phase[s] == 1 && q == 1;
+        r.has_prefill |= phase[s] == 0 || q > 1;
         const int32_t nb = (c + bs - 1) / bs;
         if (nb > block_table_stride) return FNPU_EINVAL;
+        const int32_t *row = block_table + static_cast<int64_t>(s) * block_table_stride;
+        int32_t lo = INT32_MAX, hi = INT32_MIN;  // (a min/max pass over the row vectorises)
         for (int32_t j = 0; j < nb; ++j) {
-            const int32_t b = block_table[static_cast<int64_t>(s) * block_table_stride + j];
-            if (b < 0 || b >= desc->num_blocks) return FNPU_EINVAL;
+            lo = std::min(lo, row[j]);
+            hi = std::max(hi, row[j]);
         }
-        width = std::max(width, nb);
-        T += q;
+        if (nb > 0 && (lo < 0 || hi >= desc->num_blocks)) return FNPU_EINVAL;
+        r.width = std::max(r.width, nb);
+        r.T += q;
     }
-    if (T > INT32_MAX) return FNPU_EINVAL;
+    if (r.T > INT32_MAX) return FNPU_EINVAL;
     if (num_seqs > 0) {
-        const int ks = kernel_support(desc, has_decode, has_prefill);
+        const int ks = kernel_support(desc, r.has_decode, r.has_prefill);
         if (ks != FNPU_OK) return ks;
     }
+    *m = r;
+    return FNPU_OK;
+}
 
+int plan_sms(const fnpu_plan_opts &o, int *sms) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return FNPU_ECUDA;
-    int sms = o.num_sms;
-    if (sms == 0 && cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    *sms = o.num_sms;
+    if (*sms == 0 && cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return FNPU_ECUDA;
+    return FNPU_OK;
+}
 
-    fnpu_plan *pl = new (std::nothrow) fnpu_plan();
-    if (!pl) return FNPU_ENOMEM;
+// Build (or rebuild) the work list of a validated step into `pl`, reusing
+// whatever streams, events, staging buffers and workspace it already holds.
+// On an error after validation the plan must be re-planned or destroyed.
+int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const int32_t *query_len,
+              const int32_t *context_len, const uint8_t *phase, const int32_t *block_table,
+              int32_t block_table_stride, const fnpu_plan_opts &o, const StepMeta &meta, int sms,
+              void *stream) {
+    const int32_t bs = desc->block_size;
+    const int64_t T = meta.T;
+    const int32_t width = meta.width;
     pl->desc = *desc;
     pl->scale = desc->softmax_scale > 0.f ? desc->softmax_scale
                                           : static_cast<float>(1.0 / sqrt(static_cast<double>(desc->head_dim_qk)));
     pl->num_seqs = num_seqs;
+    pl->num_jobs = 0;  // (FP8 staging, set below when the plan has some)
+    pl->tbt_width = 1;
+    pl->num_tblocks = 0;
     pl->num_tokens = T;
     pl->bt_width = width;
     pl->num_sms = sms;
@@ -623,10 +742,13 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
                               ? std::min(sms - 1, std::max(1, (sms * o.decode_share_pct + 50) / 100))
                               : choose_decode_sms(item_tiles, tile_scale, dec_bytes, sms);
         pl->pre_ctas = sms - k;
-        if (o.flags & FNPU_PLAN_GREEN_CONTEXTS) {
+        if ((o.flags & FNPU_PLAN_GREEN_CONTEXTS) && pl->g_pre && pl->green_k == k) {
+            pl->pre_ctas = pl->green_pre;  // the partitions of the last plan fit this share
+        } else if (o.flags & FNPU_PLAN_GREEN_CONTEXTS) {
             // enforce the split in hardware: a green context of at least k SMs
             // (rounded up to the partition granularity) for decode and one of
             // the remaining SMs for prefill, each with its own stream
+            destroy_streams(pl);
             const GreenApi &g = green_api();
             int dev = 0;
             CUdevice cudev = 0;
@@ -648,12 +770,14 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
             pl->s_pre = reinterpret_cast<cudaStream_t>(st_pre);
             if (!made) {
                 cudaGetLastError();
-                destroy_sync_objects(pl);
-                delete pl;
+                destroy_streams(pl);
                 return FNPU_EUNSUPPORTED;
             }
             pl->dec_sms = static_cast<int32_t>(part.sm.smCount);
-            pl->pre_ctas = static_cast<int32_t>(rest.sm.smCount);
+            pl->pre_ctas = pl->green_pre = static_cast<int32_t>(rest.sm.smCount);
+            pl->green_k = k;
+        } else if (pl->g_pre) {
+            destroy_streams(pl);  // plain streams are made below
         }
     }
     int32_t pparts = 0, pgroups = 0;
@@ -711,9 +835,15 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     std::vector<PrefillItem> pordered;
     pordered.reserve(pitems.size());
     for (auto &pc : pcost) pordered.push_back(pitems[pc.second]);
-    std::stable_sort(ditems.begin(), ditems.end(), [](const DecodeItem &a, const DecodeItem &b) {
-        return (a.key_end - a.key_begin) > (b.key_end - b.key_begin);
-    });
+    {  // (sorted through keys: the items are 64 bytes each)
+        std::vector<std::pair<int32_t, int32_t>> key(ditems.size());
+        for (size_t i = 0; i < ditems.size(); ++i)
+            key[i] = {-(ditems[i].key_end - ditems[i].key_begin), static_cast<int32_t>(i)};
+        std::sort(key.begin(), key.end());  // (length, index): the same order as a stable sort by length
+        std::vector<DecodeItem> sorted(ditems.size());
+        for (size_t i = 0; i < key.size(); ++i) sorted[i] = ditems[key[i].second];
+        ditems.swap(sorted);
+    }
 
     std::stable_sort(mitems.begin(), mitems.end(), [](const MlaItem &a, const MlaItem &b) {
         return (a.key_end - a.key_begin) > (b.key_end - b.key_begin);
@@ -727,24 +857,26 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->num_pparts = pparts;
     pl->num_pgroups = pgroups;
     if (pl->coloc) {
+        // made once per plan and kept across re-plans (green streams above)
         int lo = 0, hi = 0;
-        const bool green = pl->g_pre != nullptr;  // streams already made in the partitions
-        if (cudaDeviceGetStreamPriorityRange(&lo, &hi) != cudaSuccess ||
-            (!green && cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess) ||
-            (!green && cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess) ||
-            cudaEventCreateWithFlags(&pl->e_fork, cudaEventDefault) != cudaSuccess ||
-            cudaEventCreateWithFlags(&pl->e_started, cudaEventDisableTiming) != cudaSuccess ||
-            cudaEventCreateWithFlags(&pl->e_pre, cudaEventDefault) != cudaSuccess ||
-            cudaEventCreateWithFlags(&pl->e_dec, cudaEventDefault) != cudaSuccess) {
+        const bool mk_streams = !pl->s_pre;
+        if ((mk_streams && cudaDeviceGetStreamPriorityRange(&lo, &hi) != cudaSuccess) ||
+            (mk_streams && cudaStreamCreateWithPriority(&pl->s_pre, cudaStreamNonBlocking, hi) != cudaSuccess) ||
+            (mk_streams && cudaStreamCreateWithPriority(&pl->s_dec, cudaStreamNonBlocking, lo) != cudaSuccess) ||
+            (!pl->e_fork && cudaEventCreateWithFlags(&pl->e_fork, cudaEventDefault) != cudaSuccess) ||
+            (!pl->e_started && cudaEventCreateWithFlags(&pl->e_started, cudaEventDisableTiming) != cudaSuccess) ||
+            (!pl->e_pre && cudaEventCreateWithFlags(&pl->e_pre, cudaEventDefault) != cudaSuccess) ||
+            (!pl->e_dec && cudaEventCreateWithFlags(&pl->e_dec, cudaEventDefault) != cudaSuccess)) {
             cudaGetLastError();
-            destroy_sync_objects(pl);
-            delete pl;
             return FNPU_ECUDA;
         }
     }
 
-    // workspace: metadata (uploaded) then scratch (never read before written)
+    // workspace: the error flag and work queues (kept across re-plans), the
+    // metadata (uploaded), then scratch (never read before written)
     size_t off = 0;
+    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
+    const size_t o_meta = off;
     const size_t o_seqs = off; off = align_up(off + sizeof(SeqInfo) * std::max(num_seqs, 1), 256);
     const size_t o_bt = off; off = align_up(off + sizeof(int32_t) * static_cast<size_t>(std::max(num_seqs, 1)) * width, 256);
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
@@ -755,7 +887,6 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
     const size_t o_jobs = off; off = align_up(off + sizeof(Fp8StageJob) * std::max<size_t>(jobs.size(), 1), 256);
     const size_t o_tbt = off; off = align_up(off + sizeof(int32_t) * std::max<size_t>(tbt.size(), 1), 256);
-    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
     const size_t meta_bytes = off;
     // query heads per partial
     const int32_t part_rows = pl->use_mla_tc ? desc->num_q_heads
@@ -773,21 +904,61 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     off = align_up(off + (pl->num_jobs ? static_cast<size_t>(T) * desc->num_q_heads * desc->head_dim_qk * 2 : 0), 256);
     pl->ws_bytes = off;
 
-    if (cudaMalloc(&pl->d_ws, pl->ws_bytes) != cudaSuccess) {
-        cudaGetLastError();
-        destroy_sync_objects(pl);
-        delete pl;
-        return FNPU_ENOMEM;
+    // device workspace: allocated once, grown only when a re-plan needs more
+    // (after the work already queued on the device has finished)
+    int32_t carried_err = 0;
+    bool fresh = false;
+    if (pl->ws_bytes > pl->ws_cap) {
+        const bool growing = pl->d_ws != nullptr;
+        if (growing) {
+            if (cudaDeviceSynchronize() != cudaSuccess ||
+                cudaMemcpy(&carried_err, pl->d_ws, sizeof(int32_t), cudaMemcpyDeviceToHost) != cudaSuccess) {
+                cudaGetLastError();
+                return FNPU_ECUDA;
+            }
+            cudaFree(pl->d_ws);
+            pl->d_ws = nullptr;
+            pl->ws_cap = 0;
+        }
+        const size_t cap = growing ? pl->ws_bytes + pl->ws_bytes / 4 : pl->ws_bytes;
+        if (cudaMalloc(&pl->d_ws, cap) != cudaSuccess) {
+            cudaGetLastError();
+            pl->d_ws = nullptr;
+            return FNPU_ENOMEM;
+        }
+        pl->ws_cap = cap;
+        fresh = true;
     }
-    if (cudaMallocHost(&pl->h_stage, meta_bytes) != cudaSuccess) {
+    // pinned staging: two buffers in turn; wait (if at all) only for the
+    // upload that last used this one
+    const int turn = pl->stage_turn;
+    if (pl->e_upload[turn] && cudaEventSynchronize(pl->e_upload[turn]) != cudaSuccess) {
         cudaGetLastError();
-        cudaFree(pl->d_ws);
-        destroy_sync_objects(pl);
-        delete pl;
-        return FNPU_ENOMEM;
+        return FNPU_ECUDA;
     }
-    uint8_t *h = static_cast<uint8_t *>(pl->h_stage);
-    memset(h, 0, meta_bytes);
+    if (pl->stage_cap[turn] < meta_bytes) {
+        if (pl->h_stage[turn]) cudaFreeHost(pl->h_stage[turn]);
+        pl->h_stage[turn] = nullptr;
+        pl->stage_cap[turn] = 0;
+        const size_t cap = meta_bytes + meta_bytes / 4;
+        if (cudaMallocHost(&pl->h_stage[turn], cap) != cudaSuccess) {
+            cudaGetLastError();
+            pl->h_stage[turn] = nullptr;
+            return FNPU_ENOMEM;
+        }
+        pl->stage_cap[turn] = cap;
+    }
+    if (!pl->e_upload[turn] && cudaEventCreateWithFlags(&pl->e_upload[turn], cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        return FNPU_ECUDA;
+    }
+    uint8_t *h = static_cast<uint8_t *>(pl->h_stage[turn]);
+    // only the error flag and work queues and the merge counters must start at
+    // zero; every other region is written below where a kernel reads it (the
+    // block-table columns past a sequence's blocks are never read)
+    memset(h + o_err, 0, o_meta - o_err);
+    memset(h + o_cnt, 0, o_jobs - o_cnt);
+    reinterpret_cast<int32_t *>(h + o_err)[0] = carried_err;
     if (num_seqs) memcpy(h + o_seqs, seqs.data(), sizeof(SeqInfo) * num_seqs);
     for (int32_t s = 0; s < num_seqs; ++s)
         memcpy(h + o_bt + sizeof(int32_t) * static_cast<size_t>(s) * width,
@@ -819,17 +990,65 @@ int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const 
     pl->d_tk = d + o_tk;
     pl->d_tv = d + o_tv;
     pl->d_tq = d + o_tq;
-    if (cudaMemcpyAsync(pl->d_ws, pl->h_stage, meta_bytes, cudaMemcpyHostToDevice,
-                        static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+    // a fresh workspace gets its error flag and queues (zero) with the
+    // metadata; a reused one keeps them (the queues are zero between runs)
+    const size_t up0 = fresh ? o_err : o_meta;
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(d + up0, h + up0, meta_bytes - up0, cudaMemcpyHostToDevice, cs) != cudaSuccess ||
+        cudaEventRecord(pl->e_upload[turn], cs) != cudaSuccess) {
         cudaGetLastError();
-        cudaFreeHost(pl->h_stage);
-        cudaFree(pl->d_ws);
-        destroy_sync_objects(pl);
-        delete pl;
         return FNPU_ECUDA;
+    }
+    pl->stage_turn = turn ^ 1;
+    return FNPU_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int fnpu_mixed_attn_plan_ex(const fnpu_attn_desc *desc, int32_t num_seqs, const int32_t *query_len,
+                            const int32_t *context_len, const uint8_t *phase,
+                            const int32_t *block_table, int32_t block_table_stride,
+                            const fnpu_plan_opts *opts, void *stream, fnpu_plan **out) {
+    if (!out) return FNPU_EINVAL;
+    fnpu_plan_opts o = {};
+    if (opts) o = *opts;
+    StepMeta m;
+    int rc = validate_meta(desc, num_seqs, query_len, context_len, phase, block_table, block_table_stride, o, &m);
+    if (rc != FNPU_OK) return rc;
+    int sms = 0;
+    rc = plan_sms(o, &sms);
+    if (rc != FNPU_OK) return rc;
+    fnpu_plan *pl = new (std::nothrow) fnpu_plan();
+    if (!pl) return FNPU_ENOMEM;
+    rc = plan_fill(pl, desc, num_seqs, query_len, context_len, phase, block_table, block_table_stride, o, m, sms,
+                   stream);
+    if (rc != FNPU_OK) {
+        release_plan(pl);
+        delete pl;
+        return rc;
     }
     *out = pl;
     return FNPU_OK;
+}
+
+int fnpu_mixed_attn_replan(fnpu_plan *pl, int32_t num_seqs, const int32_t *query_len, const int32_t *context_len,
+                           const uint8_t *phase, const int32_t *block_table, int32_t block_table_stride,
+                           const fnpu_plan_opts *opts, void *stream) {
+    if (!pl) return FNPU_EINVAL;
+    fnpu_plan_opts o = {};
+    if (opts) o = *opts;
+    StepMeta m;
+    int rc = validate_meta(&pl->desc, num_seqs, query_len, context_len, phase, block_table, block_table_stride, o,
+                           &m);
+    if (rc != FNPU_OK) return rc;  // the plan is unchanged
+    int sms = 0;
+    rc = plan_sms(o, &sms);
+    if (rc != FNPU_OK) return rc;
+    const fnpu_attn_desc desc = pl->desc;
+    return plan_fill(pl, &desc, num_seqs, query_len, context_len, phase, block_table, block_table_stride, o, m, sms,
+                     stream);
 }
 
 int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache, const void *v_cache,
@@ -939,9 +1158,7 @@ int fnpu_plan_check(const fnpu_plan *pl, void *stream) {
 void fnpu_plan_destroy(fnpu_plan *pl) {
     if (!pl) return;
     cudaDeviceSynchronize();
-    destroy_sync_objects(pl);
-    if (pl->h_stage) cudaFreeHost(pl->h_stage);
-    if (pl->d_ws) cudaFree(pl->d_ws);
+    release_plan(pl);
     delete pl;
 }
 
@@ -954,7 +1171,7 @@ int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_
     if (launches_per_run)
         *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0) + (pl->num_mgroups > 0) +
                             (pl->num_jobs > 0 ? 1 : 0);  // FP8 staging: blocks and queries to f16
-    if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_bytes);
+    if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_cap);
     return FNPU_OK;
 }
 

@@ -51,8 +51,6 @@ namespace {
 constexpr int kThreads = 384;
 constexpr int kRows = 128;
 constexpr int kKeys = 128;   // keys per tile
-constexpr int kKStages = 3;  // K ring
-constexpr int kVStages = 2;  // V ring
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p <= 2^8 before a rescale
 // Register split (setmaxnreg): the softmax warpgroups hold a 128-score row
@@ -64,14 +62,21 @@ static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsHelper <= 65536 / kThreads / 8
 __host__ __device__ constexpr uint32_t col_s(int w) { return 128u * w; }
 __host__ __device__ constexpr uint32_t col_o(int w) { return 256u + 128u * w; }
 
-template <int D>
+// DQ: key (and query) width, DV: value width. 128-wide keys take a 3-stage K
+// ring and a 2-stage V ring; 192-wide keys (MLA rows expanded per head) leave
+// shared memory for 2 K stages and 1 V stage beside the two Q tiles.
+template <int DQ, int DV>
 struct TcCfg {
-    static constexpr int kTileBytes = kKeys * D * 2;  // one K or V tile
-    static constexpr int kHalf = kKeys * 128;         // one 64-column half of a K/V tile
-    static constexpr int kQHalf = kRows * 128;        // one 64-column half of a Q tile
-    static constexpr int kQBytes = kRows * D * 2;     // one Q tile
-    static constexpr int kVOff = kKStages * kTileBytes;
-    static constexpr int kQOff = kVOff + kVStages * kTileBytes;
+    static_assert(DQ % 64 == 0 && DV % 64 == 0 && DV <= 128, "tile widths");
+    static constexpr int kKStages = DQ > 128 ? 2 : 3;  // K ring
+    static constexpr int kVStages = DQ > 128 ? 1 : 2;  // V ring
+    static constexpr int kKTileBytes = kKeys * DQ * 2;  // one K tile
+    static constexpr int kVTileBytes = kKeys * DV * 2;  // one V tile
+    static constexpr int kHalf = kKeys * 128;           // one 64-column chunk of a K/V tile
+    static constexpr int kQHalf = kRows * 128;          // one 64-column chunk of a Q tile
+    static constexpr int kQBytes = kRows * DQ * 2;      // one Q tile
+    static constexpr int kVOff = kKStages * kKTileBytes;
+    static constexpr int kQOff = kVOff + kVStages * kVTileBytes;
     static constexpr int kBarOff = kQOff + 2 * kQBytes;
     // kfull[3] kempty[3] vfull[2] vempty[2] sfull[2] pfull[2] odone[2] ofree[2]
     // qfull qempty vzero itemfull[2] itemempty[2] drain
@@ -114,10 +119,11 @@ __device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
 
 // F16: the operands (Q, K, V and P) are f16 instead of bf16 (the FP8 cache's
 // prefill: its codes are dequantised to f16 first)
-template <int D, bool F16>
+template <int DQ, int DV, bool F16>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_tc_kernel(const AttnParams p, const __grid_constant__ TcMaps maps) {
-    using Cfg = TcCfg<D>;
+    using Cfg = TcCfg<DQ, DV>;
+    constexpr int kKStages = Cfg::kKStages, kVStages = Cfg::kVStages;
     extern __shared__ __align__(1024) uint8_t smem[];
     const uint32_t s_base = smem_u32(smem);
     const uint32_t s_bars = s_base + Cfg::kBarOff;
@@ -231,11 +237,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int q0 = __shfl_sync(0xffffffffu, it.q_start + it.p0, 0);
             auto load_q = [&]() -> bool {
                 if (k >= 1 && !wait(QEMPTY, (k - 1) & 1)) return false;
-                tc::mbar_arrive_expect_tx_warp(QFULL, static_cast<uint32_t>(2 * (D / 64) * 64 * G * P * 2));
+                tc::mbar_arrive_expect_tx_warp(QFULL, static_cast<uint32_t>(2 * (DQ / 64) * 64 * G * P * 2));
 #pragma unroll
                 for (int w = 0; w < 2; ++w)
 #pragma unroll
-                    for (int h = 0; h < D / 64; ++h)
+                    for (int h = 0; h < DQ / 64; ++h)
                         tc::tma_load_3d_warp(s_base + Cfg::kQOff + w * Cfg::kQBytes + h * Cfg::kQHalf, &maps.q,
                                              QFULL, h * 64, ukvh * G, q0 + w * P);
                 return true;
@@ -257,15 +263,35 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int nvalid = nblk_seq - b00 - i * per_tile;
                 nvalid = nvalid < 0 ? 0 : (nvalid > per_tile ? per_tile : nvalid);
                 nvalid = __shfl_sync(0xffffffffu, nvalid, 0);
-                const uint32_t dst = s_base + (is_k ? 0 : Cfg::kVOff) + st * Cfg::kTileBytes;
                 const uint32_t bar = is_k ? KFULL(st) : VFULL(st);
-                tc::mbar_arrive_expect_tx_warp(bar, static_cast<uint32_t>(nvalid) * bs * D * 2);
-                for (int b = 0; b < per_tile; ++b) {
-                    const int blk = __shfl_sync(0xffffffffu, blk_cur, b);
-                    if (b < nvalid) {
+                if constexpr (DQ == DV) {
+                    const uint32_t dst = s_base + (is_k ? 0 : Cfg::kVOff) + st * Cfg::kKTileBytes;
+                    tc::mbar_arrive_expect_tx_warp(bar, static_cast<uint32_t>(nvalid) * bs * DQ * 2);
+                    for (int b = 0; b < per_tile; ++b) {
+                        const int blk = __shfl_sync(0xffffffffu, blk_cur, b);
+                        if (b < nvalid) {
 #pragma unroll
-                        for (int h = 0; h < D / 64; ++h)
-                            tc::tma_load_4d_warp(dst + h * Cfg::kHalf + b * bs * 128, map, bar, h * 64, ukvh, 0, blk);
+                            for (int h = 0; h < DQ / 64; ++h)
+                                tc::tma_load_4d_warp(dst + h * Cfg::kHalf + b * bs * 128, map, bar, h * 64, ukvh, 0, blk);
+                        }
+                    }
+                } else {
+                    const uint32_t dst = s_base + (is_k ? st * Cfg::kKTileBytes : Cfg::kVOff + st * Cfg::kVTileBytes);
+                    const int dcols = is_k ? DQ : DV;
+                    tc::mbar_arrive_expect_tx_warp(bar, static_cast<uint32_t>(nvalid) * bs * dcols * 2);
+                    for (int b = 0; b < per_tile; ++b) {
+                        const int blk = __shfl_sync(0xffffffffu, blk_cur, b);
+                        if (b < nvalid) {
+                            if (is_k) {
+#pragma unroll
+                                for (int h = 0; h < DQ / 64; ++h)
+                                    tc::tma_load_4d_warp(dst + h * Cfg::kHalf + b * bs * 128, map, bar, h * 64, ukvh, 0, blk);
+                            } else {
+#pragma unroll
+                                for (int h = 0; h < DV / 64; ++h)
+                                    tc::tma_load_4d_warp(dst + h * Cfg::kHalf + b * bs * 128, map, bar, h * 64, ukvh, 0, blk);
+                            }
+                        }
                     }
                 }
                 if (!is_k && i == it.ntiles - 1 && it.tail_fix) {
@@ -273,10 +299,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!wait(VFULL(st), (g / nst) & 1)) { ok = false; break; }
                     const int r0 = it.ctx - (it.kt0 + i) * kKeys;
                     const int nrows = kKeys - r0;
-                    for (int e = lane; e < nrows * 8 * (D / 64); e += 32) {
+                    for (int e = lane; e < nrows * 8 * (DV / 64); e += 32) {
                         const int h = e / (nrows * 8), rem = e % (nrows * 8);
                         const int row = r0 + rem / 8, ch = rem % 8;
-                        *reinterpret_cast<uint4 *>(smem + Cfg::kVOff + st * Cfg::kTileBytes + h * Cfg::kHalf +
+                        *reinterpret_cast<uint4 *>(smem + Cfg::kVOff + st * Cfg::kVTileBytes + h * Cfg::kHalf +
                                                    row * 128 + ch * 16) = make_uint4(0u, 0u, 0u, 0u);
                     }
                     tc::fence_proxy_async_smem();
@@ -294,18 +320,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         // so the compiler keeps them in uniform registers); each tcgen05
         // instruction is issued by one elected lane.
         constexpr uint32_t idS = F16 ? tc::idesc_f16(kRows, kKeys, false) : tc::idesc_bf16(kRows, kKeys, false);
-        constexpr uint32_t idO = F16 ? tc::idesc_f16(kRows, D, true) : tc::idesc_bf16(kRows, D, true);
+        constexpr uint32_t idO = F16 ? tc::idesc_f16(kRows, DV, true) : tc::idesc_bf16(kRows, DV, true);
         const uint32_t utmem = __shfl_sync(0xffffffffu, tmem, 0);
         const uint32_t us_base = __shfl_sync(0xffffffffu, s_base, 0);
         int gk = 0, gv = 0, t = 0, nfix = 0;
         bool ok = true, issued = false;
         auto issue_s = [&](int w, int st_in) {
             const int st = __shfl_sync(0xffffffffu, st_in, 0);
-            const uint64_t kd = tc::sdesc_sw128(us_base + st * Cfg::kTileBytes, 16, 1024);
+            const uint64_t kd = tc::sdesc_sw128(us_base + st * Cfg::kKTileBytes, 16, 1024);
             const uint64_t qd = tc::sdesc_sw128(us_base + Cfg::kQOff + w * Cfg::kQBytes, 16, 1024);
             const uint32_t dS = utmem + col_s(w);
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk)
+            for (int kk = 0; kk < DQ / 16; ++kk)
                 tc::mma_ss_warp(dS, qd + ((kk / 4) * Cfg::kQHalf + (kk % 4) * 32) / 16,
                                 kd + ((kk / 4) * Cfg::kHalf + (kk % 4) * 32) / 16, idS, kk > 0);
             tc::commit_warp(SFULL(w));
@@ -315,7 +341,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int st = __shfl_sync(0xffffffffu, st_in, 0);
             const uint32_t acc = __shfl_sync(0xffffffffu, acc_in, 0);
             const uint64_t vd =
-                tc::sdesc_sw128(us_base + Cfg::kVOff + st * Cfg::kTileBytes, Cfg::kHalf, 1024);
+                tc::sdesc_sw128(us_base + Cfg::kVOff + st * Cfg::kVTileBytes, Cfg::kHalf, 1024);
             const uint32_t dO = utmem + col_o(w), aP = utmem + col_s(w);
             tc::mma_ts_warp(dO, aP, vd, idO, acc);
 #pragma unroll
@@ -446,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (i > 0) {
                         // PV_w(i - 1) is complete: S_w(i) was issued after it
 #pragma unroll
-                        for (int c = 0; c < D / 32; ++c) {
+                        for (int c = 0; c < DV / 32; ++c) {
                             uint32_t o[32];
                             tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
                             tc::tmem_wait_ld();
@@ -492,10 +518,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::fence_after_sync();
             const float inv = 1.f / l;
             uint4 *orow = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
-                                                    (tok * p.num_q_heads + head) * D);
+                                                    (tok * p.num_q_heads + head) * DV);
             if (it.ns == 1) {
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
+                for (int c = 0; c < DV / 32; ++c) {
                     uint32_t o[32];
                     tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
                     tc::tmem_wait_ld();
@@ -519,9 +545,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // column q in position q * 128 + r, so that a warp's stores
                 // and loads are contiguous
                 const int64_t prow = (static_cast<int64_t>(it.pbase + it.split) * 2 + w) * 128;
-                float4 *po = reinterpret_cast<float4 *>(p.ppart_o) + prow * (D / 4) + r;
+                float4 *po = reinterpret_cast<float4 *>(p.ppart_o) + prow * (DV / 4) + r;
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
+                for (int c = 0; c < DV / 32; ++c) {
                     uint32_t o[32];
                     tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
                     tc::tmem_wait_ld();
@@ -551,7 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int sp = 0; sp < it.ns; ++sp) L += fast_exp2((sp == it.split ? my_lse : lse_of(sp)) - M);
                     const float iL = 1.f / L;
 #pragma unroll 1
-                    for (int c = 0; c < D / 32; ++c) {
+                    for (int c = 0; c < DV / 32; ++c) {
                         uint32_t o[32];
                         tc::tmem_ld32(lane_addr + col_o(w) + 32 * c, o);
                         tc::tmem_wait_ld();
@@ -570,7 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             } else {
                                 ws = fast_exp2(lse_of(sp) - M);
                                 const float4 *q4 = reinterpret_cast<const float4 *>(p.ppart_o) +
-                                                   (static_cast<int64_t>(it.pbase + sp) * 2 + w) * 128 * (D / 4) + r;
+                                                   (static_cast<int64_t>(it.pbase + sp) * 2 + w) * 128 * (DV / 4) + r;
 #pragma unroll
                                 for (int j = 0; j < 8; ++j) v[j] = __ldcg(q4 + (c * 8 + j) * 128);
                             }
@@ -651,28 +677,30 @@ bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, in
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D, bool F16>
+template <int DQ, int DV, bool F16>
 int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t started) {
-    using Cfg = TcCfg<D>;
+    using Cfg = TcCfg<DQ, DV>;
     TcMaps maps;
-    if (!encode_cache_map(&maps.k, p.k_cache, D, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
-        !encode_cache_map(&maps.v, p.v_cache, D, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
-        !encode_q_map(&maps.q, p.q, D, p.num_q_heads, p.num_tokens, p.group, kRows / p.group, F16))
+    if (!encode_cache_map(&maps.k, p.k_cache, DQ, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
+        !encode_cache_map(&maps.v, p.v_cache, DV, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
+        !encode_q_map(&maps.q, p.q, DQ, p.num_q_heads, p.num_tokens, p.group, kRows / p.group, F16))
         return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
-    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D, F16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Cfg::kSmemBytes));
-    FNPU_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<D, F16>, cudaFuncAttributePreferredSharedMemoryCarveout,
+    auto kernel = prefill_tc_kernel<DQ, DV, F16>;
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes));
+    FNPU_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                                        cudaSharedmemCarveoutMaxShared));
     const int grid = p.num_pitems < max_ctas ? p.num_pitems : max_ctas;
-    FNPU_CUDA_TRY(launch_ex(prefill_tc_kernel<D, F16>, grid, kThreads, Cfg::kSmemBytes, st, false, started, p, maps));
+    FNPU_CUDA_TRY(launch_ex(kernel, grid, kThreads, Cfg::kSmemBytes, st, false, started, p, maps));
     return FNPU_OK;
 }
 
 }  // namespace
 
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group) {
-    return d_qk == d_v && (d_qk == 64 || d_qk == 128) &&
-           (block_size == 16 || block_size == 32 || block_size == 64) && group >= 1 && group <= kRows;
+    // split K/V heads of 64 or 128; the per-head keys (192) and values (128)
+    // of an expanded latent cache, one kv head per query head
+    const bool dims = (d_qk == d_v && (d_qk == 64 || d_qk == 128)) || (d_qk == 192 && d_v == 128 && group == 1);
+    return dims && (block_size == 16 || block_size == 32 || block_size == 64) && group >= 1 && group <= kRows;
 }
 
 // positions per work item: two Q tiles of floor(128 / G) positions each
@@ -685,12 +713,15 @@ int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *sta
     if (p.num_pitems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaEvent_t ev = static_cast<cudaEvent_t>(started);
-    if (f16) return p.head_dim_qk == 128 ? launch_tc<128, true>(p, st, max_ctas, ev) : FNPU_EUNSUPPORTED;
-    switch (p.head_dim_qk) {
-        case 64: return launch_tc<64, false>(p, st, max_ctas, ev);
-        case 128: return launch_tc<128, false>(p, st, max_ctas, ev);
-        default: return FNPU_EUNSUPPORTED;
-    }
+    if (f16)
+        return p.head_dim_qk == 128 && p.head_dim_v == 128 ? launch_tc<128, 128, true>(p, st, max_ctas, ev)
+                                                            : FNPU_EUNSUPPORTED;
+    if (p.head_dim_qk == 64 && p.head_dim_v == 64) return launch_tc<64, 64, false>(p, st, max_ctas, ev);
+    if (p.head_dim_qk == 128 && p.head_dim_v == 128)
+        return launch_tc<128, 128, false>(p, st, max_ctas, ev);
+    if (p.head_dim_qk == 192 && p.head_dim_v == 128)
+        return launch_tc<192, 128, false>(p, st, max_ctas, ev);
+    return FNPU_EUNSUPPORTED;
 }
 
 }  // namespace fnpu

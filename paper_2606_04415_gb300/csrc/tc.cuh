@@ -124,6 +124,15 @@ __device__ __forceinline__ void tma_load_4d_warp(uint32_t dst, const CUtensorMap
         "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
         : "memory");
 }
+__device__ __forceinline__ void tma_load_2d_warp(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
+                                                 int c1) {
+    asm volatile(
+        "{\n .reg .pred p;\n elect.sync _|p, 0xffffffff;\n"
+        " @p cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];\n}\n" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
+        : "memory");
+}
 __device__ __forceinline__ void tma_load_3d_warp(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
                                                  int c1, int c2) {
     asm volatile(
@@ -132,6 +141,19 @@ __device__ __forceinline__ void tma_load_3d_warp(uint32_t dst, const CUtensorMap
         " [%0], [%1, {%3, %4, %5}], [%2];\n}\n" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
         : "memory");
+}
+// TMA tiled store shared -> global of one box (the elected lane issues it),
+// tracked by the bulk async-group of the issuing thread.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t src, int c0, int c1, int c2) {
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4}], [%1];\n" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(src), "r"(c0), "r"(c1), "r"(c2)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit_group() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
+// wait until the shared-memory sources of this thread's bulk stores are read
+__device__ __forceinline__ void bulk_wait_group_read0() {
+    asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory");
 }
 // Warp-collective untiled bulk copy global -> shared (both addresses 16-byte
 // aligned, size a multiple of 16), completing on mbarrier `bar`.

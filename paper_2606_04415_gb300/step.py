@@ -17,7 +17,8 @@ from typing import Optional
 
 import numpy as np
 
-from . import (FP8_BLOCK_BYTES, PlanOpts, kv_append, make_desc, mixed_attn_plan, mixed_attn_run)
+from . import (FP8_BLOCK_BYTES, PlanOpts, kv_append, make_desc, mixed_attn_plan, mixed_attn_replan,
+               mixed_attn_run)
 
 
 def _to_dev(a: Optional[np.ndarray], torch, dtype, device):
@@ -79,12 +80,12 @@ class DeviceStep:
         kv_append(self.desc, _to_dev(k, torch, torch.bfloat16, device), _to_dev(v, torch, torch.bfloat16, device),
                   _to_dev(sl, torch, None, device), self.k_cache, self.v_cache)
 
-    def replan(self, opts: Optional[PlanOpts] = None):
+    def replan(self, opts: Optional[PlanOpts] = None, stream=None):
         """Plan the same batch again with other options (for instance the
-        decode share a dispatch controller chose for the next step)."""
-        self.plan.destroy()
+        decode share a dispatch controller chose for the next step), reusing
+        the plan's resources (``fnpu_mixed_attn_replan``)."""
         b = self.batch
-        self.plan = mixed_attn_plan(self.desc, b.query_len, b.context_len, b.phase, b.block_table, opts=opts)
+        mixed_attn_replan(self.plan, b.query_len, b.context_len, b.phase, b.block_table, opts=opts, stream=stream)
 
     def append(self, stream=None):
         kv_append(self.desc, self.k_new, self.v_new, self.slot_mapping, self.k_cache, self.v_cache,

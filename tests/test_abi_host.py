@@ -121,6 +121,7 @@ def test_append_and_run_reject_null_pointers():
     assert rc == fnpu.FNPU_EINVAL
     assert lib.fnpu_mixed_attn_run(None, None, None, None, None, None, None) == fnpu.FNPU_EINVAL
     assert lib.fnpu_plan_check(None, None) == fnpu.FNPU_EINVAL
+    assert lib.fnpu_mixed_attn_replan(None, 0, None, None, None, None, 1, None, None) == fnpu.FNPU_EINVAL
     lib.fnpu_plan_destroy(None)  # ignored
 
 

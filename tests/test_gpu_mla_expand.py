@@ -1,7 +1,8 @@
 """MLA prefill without absorption on the GPU: latent rows expanded into
-per-head keys and values (fnpu_mla_expand: the library's gather kernel and two
-cuBLAS GEMMs), then multi-head attention (d_qk 192, d_v 128) over them through
-the plan / run, against the fp64 reference (oracle.mla_expand + the C oracle).
+per-head keys and values (fnpu_mla_expand), then multi-head attention (d_qk
+192, d_v 128) over them through the plan / run (the tcgen05 prefill kernel,
+or the mma.sync one under FNPU_PLAN_NO_TCGEN05), against the fp64 reference
+(oracle.mla_expand + the C oracle).
 
 Expanded rows: the rotary part is a copy (bit-exact); the products are fp32
 sums rounded to bf16 against the reference's exactly rounded fp64 sums, so an
@@ -83,7 +84,7 @@ def _expansion_bounds(batch, bt, q_bits, gk, gv, kb, vb, toks):
     return lse_bound, o_bound
 
 
-def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
+def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None, flags=0):
     import paper_2606_04415_gb300 as fnpu
     from paper_2606_04415_gb300.step import ExpandedMlaPrefill
     rng = np.random.default_rng(seed)
@@ -91,7 +92,8 @@ def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
     batch = W.build_batch(sh, q_lens, ctxs, [0] * len(q_lens), rng, name="mla_expand")
     ins = W.mla_expand_inputs(batch, seed)
     slots, bt, nb = W.expanded_layout(batch)
-    st = ExpandedMlaPrefill(batch, ins["w_uk"], ins["w_uv"], ins["q"], slots, bt, nb)
+    st = ExpandedMlaPrefill(batch, ins["w_uk"], ins["w_uv"], ins["q"], slots, bt, nb,
+                            opts=fnpu.PlanOpts(0, 0, 0, flags))
     st.run()
     assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK and fnpu.check() == fnpu.FNPU_OK
     out, lse = st.results()
@@ -122,17 +124,22 @@ def _run(q_lens, ctxs, heads=128, seed=0, bs=64, tokens=None):
     return st
 
 
+@pytest.mark.parametrize("flags", [0, 2])
 @pytest.mark.parametrize("seed", [0, 1])
-def test_attention_kernel_on_192_128_heads(seed):
-    """The mma.sync prefill kernel for 192-wide keys and 128-wide values, one
-    kv head per query head (the expanded MLA shape), on random bf16 caches:
-    ragged chunks on prefixes, all rows, the attention tolerances."""
+def test_attention_kernel_on_192_128_heads(seed, flags):
+    """The prefill kernels for 192-wide keys and 128-wide values, one kv head
+    per query head (the expanded MLA shape): the tcgen05 kernel (flags 0) and
+    the mma.sync one (FNPU_PLAN_NO_TCGEN05), on random bf16 caches: ragged
+    chunks on prefixes (rows and keys off every tile boundary, a 600-row
+    chunk of three 256-row items, the last one ragged), all rows, the
+    attention tolerances."""
     from paper_2606_04415_gb300.step import DeviceStep
     import paper_2606_04415_gb300 as fnpu
     rng = np.random.default_rng(60 + seed)
     sh = W.Shape(16, 16, 192, 128, 16, False)
-    batch = W.build_batch(sh, [1, 17, 64, 130], [1, 40, 364, 700], [0, 0, 0, 0], rng, name="mha192")
-    st = DeviceStep(batch)
+    batch = W.build_batch(sh, [1, 17, 64, 130, 600], [1, 40, 364, 700, 1000], [0, 0, 0, 0, 0], rng,
+                          name="mha192")
+    st = DeviceStep(batch, opts=fnpu.PlanOpts(0, 0, 0, flags))
     st.run()
     assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
     out, lse = st.results()
@@ -141,11 +148,13 @@ def test_attention_kernel_on_192_128_heads(seed):
     assert np.abs(out - ref_o).max() <= O_TOL and np.abs(lse - ref_l).max() <= LSE_TOL
 
 
+@pytest.mark.parametrize("flags", [0, 2])
 @pytest.mark.parametrize("heads", [128, 16])
-def test_ragged_chunks_on_prefixes(heads):
+def test_ragged_chunks_on_prefixes(heads, flags):
     """Chunks of 1, 17, 64 and 200 rows on prefixes of 0, 23, 300 and 824
-    (rows and keys off every tile boundary), latent blocks of 64."""
-    _run([1, 17, 64, 200], [1, 40, 364, 1024], heads=heads, seed=1)
+    (rows and keys off every tile boundary), latent blocks of 64; the tcgen05
+    and the mma.sync attention."""
+    _run([1, 17, 64, 200], [1, 40, 364, 1024], heads=heads, seed=1, flags=flags)
 
 
 def test_latent_blocks_of_16():

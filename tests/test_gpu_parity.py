@@ -525,3 +525,61 @@ def test_green_context_partitions(share):
     assert np.abs(a_out - b_out).max() <= O_TOL and np.abs(a_lse - b_lse).max() <= LSE_TOL
     pre, dec = fnpu.plan_phase_ms(st.plan)
     assert pre > 0 and dec > 0
+
+
+@pytest.mark.parametrize("flags", [0, 4])
+def test_replan_reuses_the_plan_across_steps(flags):
+    """fnpu_mixed_attn_replan: one plan re-planned for steps of other shapes
+    and decode shares (a larger step grows the workspace, a smaller one
+    reuses it; green-context partitions are rebuilt when the share asks for
+    another size), each run checked against the oracle."""
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    big = W.make_batch("qwen_coloc", seed=2)
+    # a small step over a pool of the same descriptor (a re-plan keeps the
+    # plan's descriptor: same heads, dims, block size and pool size)
+    rng = np.random.default_rng(11)
+    small = W.build_batch(W.SHAPES["qwen"], [70, 1, 1, 3], [300, 100, 500, 1000], [0, 1, 1, 1], rng,
+                          name="small", num_blocks=big.num_blocks)
+    st = DeviceStep(small, opts=fnpu.PlanOpts(0, 0, 0, flags))
+    st.run()
+    _compare(small, *st.results())
+    ws0 = st.plan.info()["workspace_bytes"]
+    sbig = DeviceStep(big, opts=fnpu.PlanOpts(0, 20, 0, flags))
+    tokens = _sample_tokens(big)
+    for share in (20, 12, 20):
+        sbig.replan(fnpu.PlanOpts(0, share, 0, flags))
+        sbig.run()  # (appending the same new rows again stores the same bits)
+        assert fnpu.plan_check(sbig.plan) == fnpu.FNPU_OK
+        _compare(big, *sbig.results(), tokens=tokens)
+    # the small plan re-planned for the big step (the workspace grows), then back
+    b = big
+    fnpu.mixed_attn_replan(st.plan, b.query_len, b.context_len, b.phase, b.block_table,
+                           opts=fnpu.PlanOpts(0, 16, 0, flags))
+    assert st.plan.info()["workspace_bytes"] > ws0
+    out = torch.empty_like(sbig.out)
+    lse = torch.empty_like(sbig.lse)
+    fnpu.mixed_attn_run(st.plan, sbig.q, sbig.k_cache, sbig.v_cache, out, lse)
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
+    torch.cuda.synchronize()
+    _compare(big, out.float().cpu().numpy(), lse.cpu().numpy(), tokens=tokens)
+    grown = st.plan.info()["workspace_bytes"]
+    st.replan(fnpu.PlanOpts(0, 0, 0, flags))
+    assert st.plan.info()["workspace_bytes"] == grown  # kept, not shrunk
+    st.attend()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
+    _compare(small, *st.results())
+
+
+def test_replan_rejects_bad_metadata_and_keeps_the_plan():
+    import paper_2606_04415_gb300 as fnpu
+    batch = W.make_batch("tiny", seed=12)
+    st = _step(batch)
+    bad_ctx = batch.context_len.copy()
+    bad_ctx[0] = batch.query_len[0] - 1  # ctx < q
+    with pytest.raises(fnpu.FnpuError) as e:
+        fnpu.mixed_attn_replan(st.plan, batch.query_len, bad_ctx, batch.phase, batch.block_table)
+    assert e.value.code == fnpu.FNPU_EINVAL
+    st.attend()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
+    _compare(batch, *st.results())
