@@ -336,8 +336,8 @@ int fnpu_version(void);
  *   k_out         device bf16 [n, Hq, 192];  v_out device bf16 [n, Hq, 128]
  * Two kernels of this library on the stream: a gather of the c parts into
  * the workspace (and of the r parts into every head's key), then one
- * tcgen05 GEMM (per CTA 256 rows x one head's 128 key and 128 value
- * columns, fp32 accumulators in tensor memory) for both products.
+ * tcgen05 GEMM (per CTA 128 rows x one head's 128 key and 128 value
+ * columns, an fp32 accumulator in tensor memory) for both products.
  * Errors: FNPU_EINVAL for NULL or misaligned pointers (16 bytes; slots 8),
  * n < 0 or a desc that is not a latent cache; FNPU_EUNSUPPORTED for other
  * latent widths; FNPU_ECUDA if a CUDA call fails. A slot >=

