@@ -49,7 +49,8 @@ L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 # summaries with the commands are under profiles/. Set to None for a
 # workload whose kernels change until they are captured again.
 NCU_TRAFFIC = {
-    "qwen_coloc": 472.4e6,       # prefill_tc 33.3 MB + decode_tma 437.7 MB read + 1.4 MB write
+    # co-located workloads: the prefill kernel (the dominant one), captured alone
+    "qwen_coloc": 33.5e6,        # prefill_tc 33.3 MB read + 0.21 MB write
     "qwen_decode": 308.9e6,      # decode_tma 308.15 MB read + 0.7 MB write
     "qwen_decode_fp8": 159.6e6,  # decode_fp8 159.16 MB read + 0.4 MB write
 }
@@ -573,7 +574,13 @@ def run_fnpu(args):
     # warm-up; with --dispatch feedback each warm-up step also feeds its phase
     # times to the decode-share controller and the next step is planned with
     # the share it returns (Sec. 3.4 dispatch ratio)
-    share = args.decode_share if args.decode_share > 0 else 24
+    # (the controller starts from the share the planner chose)
+    share = args.decode_share
+    if share <= 0:
+        try:
+            share = fnpu.plan_decode_share(st.plan)
+        except fnpu.FnpuError:  # one phase only: no share
+            share = 24
     trace = []
     for w in range(args.warmup):
         if args.dispatch == "feedback":
@@ -609,6 +616,7 @@ def run_fnpu(args):
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
+    # the timed steps: append (fnpu_kv_append) + attention (fnpu_mixed_attn_run)
     with ClockSampler(local) as clocks:
         for i in range(K):
             _flush_l2(flush, flush_r)  # evict L2 between timed steps (outside the events)
@@ -625,6 +633,22 @@ def run_fnpu(args):
     t_attn = [ev[i][1].elapsed_time(ev[i][2]) for i in range(K)]
     step_ms = max_over_ranks(sum(a + b for a, b in zip(t_append, t_attn)) / K, ws, dev)
     attn_ms = sum(t_attn) / K
+
+    # for a co-located plan, in a separate loop of K steps, the phase times of
+    # the attention call (fork to the end of the prefill kernel on its stream,
+    # and to the end of the decode kernel and merge on theirs)
+    phase = []
+    if info["launches_per_run"] >= 2 and not batch.shape.latent:
+        for i in range(K):
+            _flush_l2(flush, flush_r)
+            st.run()
+            try:
+                phase.append(fnpu.plan_phase_ms(st.plan))
+            except fnpu.FnpuError:  # not co-located
+                break
+    torch.cuda.synchronize(dev)
+    if fnpu.plan_check(st.plan) != fnpu.FNPU_OK or fnpu.check() != fnpu.FNPU_OK:
+        raise RuntimeError("device error flag raised in the timed steps")
 
     # end to end through host buffers: H2D of the step's inputs, append + attention,
     # D2H of the outputs, all inside the timed region
@@ -673,18 +697,27 @@ def run_fnpu(args):
     e2e_pipe_replan = max_over_ranks(pipelined_e2e(st, host_in, (h_o, h_l), K, args.warmup, replan_opts=share_opts),
                                      ws, dev)
 
-    # roofline of the dominant kernel work (the attention launch): algorithmic
-    # FLOPs and bytes per run / measured duration
+    # roofline of the dominant kernel: for a co-located step the prefill
+    # kernel (its tile FLOPs over the prefill phase of the step, from the fork
+    # to the end of the prefill stream), else the attention call (FLOPs and
+    # bytes per run over its duration)
     F = work["flops"]
     B_attn = work["bytes"] - work["append_bytes"] - 8 * batch.num_tokens
     t_s = attn_ms * 1e-3
     tf_time = F / (peaks["bf16_tflops"] * 1e12)
     hb_time = B_attn / (peaks["hbm_gbs"] * 1e9)
-    if tf_time >= hb_time:
+    if phase:
+        pre_ms = sum(x[0] for x in phase) / len(phase)
+        F_pre = W.prefill_path_flops(batch)
+        roof = {"bound": "tensor", "achieved": F_pre / (pre_ms * 1e-3) / 1e12, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s", "kernel": "prefill_tc_kernel (fork to the end of the prefill stream)",
+                "flops": F_pre, "ms": pre_ms}
+    elif tf_time >= hb_time:
         roof = {"bound": "tensor", "achieved": F / t_s / 1e12, "peak": peaks["bf16_tflops"],
-                "unit": "TFLOP/s"}
+                "unit": "TFLOP/s", "kernel": "the attention call"}
     else:
-        roof = {"bound": "hbm", "achieved": B_attn / t_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+        roof = {"bound": "hbm", "achieved": B_attn / t_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "kernel": "the attention call"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["traffic"] = args.traffic if args.traffic is not None else \
         NCU_TRAFFIC.get(args.workload + ("_fp8" if args.kv_fp8 else ""))
@@ -709,7 +742,9 @@ def run_fnpu(args):
         "roofline_step_frac": {"burst": step_roof / (step_ms * 1e-3),
                                "sustained": step_roof_sus / (step_ms * 1e-3),
                                "denominator": "max(F/bf16 peak, B/HBM peak) of measured"},
-        "kernel_ms": {"append": sum(t_append) / K, "attention": attn_ms},
+        "kernel_ms": {"append": sum(t_append) / K, "attention": attn_ms,
+                      "prefill_phase": (sum(x[0] for x in phase) / len(phase)) if phase else None,
+                      "decode_phase": (sum(x[1] for x in phase) / len(phase)) if phase else None},
         "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e,
                 "serial": "each step's copies up, step, copies down, one after the other; L2 flushed between steps",
@@ -719,7 +754,7 @@ def run_fnpu(args):
                                      "(copy streams, two buffer sets); no L2 flush, a step reads > L2"},
                 "pipelined_replan_every_step": {"value": job_throughput(ws, T, e2e_pipe_replan),
                                                 "ms_per_step": e2e_pipe_replan}},
-        "gpu_launches": K * (1 + info["launches_per_run"]),
+        "gpu_launches": K * (1 + info["launches_per_run"]),  # the append and the run's launches
         "clocks": clk,
     }
     if args.dispatch == "feedback":

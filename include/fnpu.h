@@ -201,6 +201,7 @@ int fnpu_mixed_attn_replan(fnpu_plan *plan, int32_t num_seqs, const int32_t *que
 int fnpu_mixed_attn_run(const fnpu_plan *plan, const void *q, const void *k_cache,
                         const void *v_cache, void *out, float *lse, void *stream);
 
+
 /* Synchronise `stream`, then read and clear the plan's device error flag:
  * FNPU_OK, FNPU_EDEVICE_TIMEOUT or FNPU_ECUDA. After FNPU_EDEVICE_TIMEOUT the
  * outputs of the failed run are undefined; the plan's work queues and split
@@ -252,6 +253,19 @@ int fnpu_plan_info(const fnpu_plan *plan, int32_t *prefill_items, int32_t *decod
 int fnpu_plan_phase_ms(const fnpu_plan *plan, float *prefill_ms, float *decode_ms);
 int fnpu_dispatch_next_share(int32_t share_pct, float prefill_ms, float decode_ms, float tolerance,
                              int32_t *next_share_pct);
+
+/*
+ * The decode share (percent of the SMs whose CTAs start on decode, rounded,
+ * at least 1) that a co-located plan uses: the one it was given, or the
+ * planner's own choice when decode_share_pct was 0. A serving loop starts its
+ * feedback from it. The planner models each prefill CTA as ending at its load
+ * of the longest-first schedule of the prefill items, and the decode as
+ * streaming on its own SMs from the start and on each prefill SM once that
+ * SM's CTA has ended; it takes the share with the shortest modelled step.
+ *   Errors: FNPU_EINVAL for NULL arguments; FNPU_EUNSUPPORTED for a plan that
+ *   does not co-locate.
+ */
+int fnpu_plan_decode_share(const fnpu_plan *plan, int32_t *share_pct);
 
 /*
  * Decode attention without any allocation. The paper has no counterpart:

@@ -42,6 +42,7 @@ EXPORTED = (
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
     "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error", "fnpu_plan_phase_ms",
     "fnpu_dispatch_next_share", "fnpu_mla_expand", "fnpu_mixed_attn_replan",
+    "fnpu_plan_decode_share",
 )
 
 
@@ -92,6 +93,7 @@ def load(build_if_missing: bool = True):
                                             ctypes.POINTER(PlanOpts), P, ctypes.POINTER(P)]
     lib.fnpu_mixed_attn_replan.argtypes = [P, i32, P, P, P, P, i32, ctypes.POINTER(PlanOpts), P]
     lib.fnpu_mixed_attn_run.argtypes = [P, P, P, P, P, P, P]
+    lib.fnpu_plan_decode_share.argtypes = [P, ctypes.POINTER(i32)]
     lib.fnpu_mla_expand.argtypes = [ctypes.POINTER(AttnDesc), P, P, i32, P, P, P, P, P, P]
     lib.fnpu_plan_check.argtypes = [P, P]
     lib.fnpu_check.argtypes = [P]
@@ -111,7 +113,8 @@ def load(build_if_missing: bool = True):
     for name in ("fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex",
                  "fnpu_mixed_attn_run", "fnpu_plan_check", "fnpu_check", "fnpu_plan_info",
                  "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_plan_phase_ms",
-                 "fnpu_dispatch_next_share", "fnpu_mla_expand", "fnpu_mixed_attn_replan"):
+                 "fnpu_dispatch_next_share", "fnpu_mla_expand", "fnpu_mixed_attn_replan",
+                 "fnpu_plan_decode_share"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -295,6 +298,15 @@ def plan_phase_ms(plan: Plan) -> tuple:
     if rc != FNPU_OK:
         raise FnpuError(rc, "fnpu_plan_phase_ms")
     return a.value, b.value
+
+
+def plan_decode_share(plan: Plan) -> int:
+    """Decode share (percent of SMs) a co-located plan uses."""
+    out = ctypes.c_int32()
+    rc = load().fnpu_plan_decode_share(plan.handle, ctypes.byref(out))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_plan_decode_share")
+    return out.value
 
 
 def dispatch_next_share(share_pct: int, prefill_ms: float, decode_ms: float, tolerance: float = 0.05) -> int:

@@ -176,29 +176,46 @@ constexpr double kTileSec = 1.5e-6;
 constexpr double kDecodeSmBps = 69e9;
 constexpr double kDecodeAllBps = 4.0e12;
 
-// (stop_at: the run may end as soon as the makespan reaches it)
-int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_at = INT64_MAX);
+// (stop_at: the run may end as soon as the makespan reaches it; loads, if
+// given, receives the final number of workers per load)
+int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_at = INT64_MAX,
+                     std::vector<int32_t> *loads = nullptr);
 std::vector<int32_t> cost_histogram(const std::vector<int64_t> &costs);
 
 // SMs that start on decode while the others run prefill: the prefill CTAs on
-// sms - k SMs take the items longest first, so they last about the LPT
-// makespan Tp of the item costs on sms - k workers (a step function of k:
-// whole items); decode streams at min(all, k * per SM) meanwhile, and what is
-// left runs on every SM once the prefill CTAs have finished. The k with the
-// shortest modelled step wins, the largest such k on ties (more decode done
-// while the prefill lasts).
+// sms - k SMs take the items longest first, so each ends at its load of the
+// LPT schedule of the item costs on sms - k workers, the last at the makespan
+// Tp. Decode streams at min(all, per SM x SMs it holds) on the k SMs from the
+// start and on each prefill SM from the moment its CTA ends (its CTAs take
+// the SMs the prefill leaves), until the decode bytes are read at Td. The k
+// with the shortest modelled step max(Tp, Td) wins, the largest such k on
+// ties (more decode done while the prefill lasts).
 int32_t choose_decode_sms(const std::vector<int64_t> &item_tiles, double tile_scale, int64_t dec_bytes,
                           int32_t sms) {
     int32_t best_k = 1;
     double best_t = -1.0;
     const std::vector<int32_t> hist = cost_histogram(item_tiles);
+    const double unit = tile_scale * kTileSec;  // seconds per cost unit
+    std::vector<int32_t> loads;
     for (int32_t k = 1; k <= sms / 2; ++k) {
-        const double tp = static_cast<double>(lpt_makespan(hist, sms - k)) * tile_scale * kTileSec;
-        const double rate = std::min(kDecodeAllBps, k * kDecodeSmBps);
-        const double left = std::max(0.0, static_cast<double>(dec_bytes) - tp * rate);
-        const double t = tp + left / kDecodeAllBps;
-        if (best_t < 0 || t <= best_t) {
-            best_t = t;
+        const double tp = static_cast<double>(lpt_makespan(hist, sms - k, INT64_MAX, &loads)) * unit;
+        double left = static_cast<double>(dec_bytes), t = 0.0;
+        int32_t n = k;
+        for (size_t ld = 0; ld <= loads.size() && left > 0.0; ++ld) {
+            // decode on n SMs until the next prefill CTAs end (at load ld)
+            const double next = ld < loads.size() ? static_cast<double>(ld) * unit : 1e30;
+            if (ld < loads.size() && loads[ld] == 0) continue;
+            const double rate = std::min(kDecodeAllBps, n * kDecodeSmBps);
+            if (next > t) {
+                const double run = std::min(next - t, left / rate);
+                left -= run * rate;
+                t += run;
+            }
+            if (ld < loads.size()) n += loads[ld];
+        }
+        const double step = std::max(tp, t);
+        if (best_t < 0 || step <= best_t) {
+            best_t = step;
             best_k = k;
         }
     }
@@ -242,14 +259,17 @@ std::vector<int32_t> cost_histogram(const std::vector<int64_t> &costs) {
 // to them together (workers are interchangeable, so the loads evolve as with
 // one item at a time). No load exceeds the mean plus the largest item, which
 // bounds the counts. Linear in distinct costs + loads.
-int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_at) {
+int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_at, std::vector<int32_t> *loads) {
     m = std::max<int32_t>(m, 1);
     int64_t total = 0, n = 0;
     for (size_t c = 0; c < hist.size(); ++c) {
         total += static_cast<int64_t>(c) * hist[c];
         n += hist[c];
     }
-    if (n == 0) return 0;
+    if (n == 0) {
+        if (loads) loads->assign(1, m);
+        return 0;
+    }
     const int64_t cmax = static_cast<int64_t>(hist.size()) - 1;
     const size_t bound = static_cast<size_t>(total / m + cmax + 1);
     thread_local std::vector<int32_t> cnt;
@@ -269,6 +289,7 @@ int64_t lpt_makespan(const std::vector<int32_t> &hist, int32_t m, int64_t stop_a
             if (span >= stop_at) return span;  // the caller only wants spans below stop_at
         }
     }
+    if (loads) loads->assign(cnt.begin(), cnt.begin() + static_cast<std::ptrdiff_t>(span) + 1);
     return span;
 }
 
@@ -322,7 +343,7 @@ std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int
     // not decrease with n, so the feasible counts are 1 .. nmax
     std::vector<int32_t> nmax(units.size(), 1);
     for (size_t i = 0; i < units.size(); ++i) {
-        int32_t n = 16;
+        int32_t n = std::min<int32_t>(16, std::max<int32_t>(units[i].ntiles, 1));  // no empty piece
         while (n > 1 && split_bound(units[i].ntiles, n, n - 1) > units[i].max_start) --n;
         nmax[i] = n;
     }
@@ -334,12 +355,25 @@ std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int
         // fraction of at least 1 / cap, above 1e-8, and the product errs by far
         // less than the 1e-9 added (the conversion truncates, = floor here)
         const double inv = 1.0 / static_cast<double>(cap);
+        // (no schedule on sms workers is shorter than ceil(total / sms), so a
+        // candidate whose total already reaches the best span is skipped)
+        // (units come in runs with equal tile counts and split limits, one
+        // per kv head of a row block: such a unit repeats the one before)
+        int64_t tot = 0;
         for (size_t i = 0; i < units.size(); ++i) {
-            const int32_t q = static_cast<int32_t>((units[i].ntiles - 1) * inv + 1e-9) + 1;
-            ns[i] = std::min(q, nmax[i]);
+            int32_t n;
+            if (i > 0 && units[i].ntiles == units[i - 1].ntiles && nmax[i] == nmax[i - 1]) {
+                n = ns[i - 1];
+            } else {
+                const int32_t q = static_cast<int32_t>((units[i].ntiles - 1) * inv + 1e-9) + 1;
+                n = std::min(q, nmax[i]);
+            }
+            ns[i] = n;
+            tot += units[i].ntiles + static_cast<int64_t>(n) * (kTcItemCost + (n > 1 ? kTcMergeCost : 0));
         }
         if (ns == prev) continue;  // the same splits as the candidate before
         prev = ns;
+        if (best_span >= 0 && (tot + sms - 1) / sms >= best_span) continue;
         std::fill(hist.begin(), hist.end(), 0);
         for (size_t i = 0; i < units.size(); ++i) {
             // n pieces of floor(ntiles / n) or one more tiles (split_bound
@@ -1071,17 +1105,15 @@ int fnpu_mixed_attn_replan(fnpu_plan *pl, int32_t num_seqs, const int32_t *query
                      stream);
 }
 
-int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache, const void *v_cache,
-                        void *out, float *lse, void *stream) {
-    if (!pl) return FNPU_EINVAL;
-    if (pl->num_tokens == 0) return FNPU_OK;
-    const bool latent = pl->desc.v_in_k_latent != 0;
-    if (!q || !k_cache || !out || !lse || (!latent && !v_cache)) return FNPU_EINVAL;
-    const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_cache) |
-                          reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(lse) |
-                          (latent ? 0 : reinterpret_cast<uintptr_t>(v_cache));
-    if (mis & 15u) return FNPU_EINVAL;
+}  // extern "C"
 
+namespace fnpu {
+namespace {
+
+// The kernels' arguments for one run of a plan (pointers checked by the caller).
+AttnParams run_params(const fnpu_plan *pl, const void *q, const void *k_cache, const void *v_cache, void *out,
+                      float *lse) {
+    const bool latent = pl->desc.v_in_k_latent != 0;
     AttnParams p = {};
     const fnpu_attn_desc &d = pl->desc;
     p.q = q;
@@ -1119,34 +1151,62 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     p.pcounters = pl->d_pcounters;
     p.err = pl->d_err;
     p.sched = pl->d_err + 2;
+    return p;
+}
 
-    if (pl->use_mla) return pl->use_mla_tc ? launch_mla_tc(p, stream) : launch_mla(p, stream);
-    if (pl->coloc) {
-        // both phases at once: pre_ctas persistent prefill CTAs (one per SM,
-        // the tensor pipe; a decode CTA does not fit beside one) and decode
-        // CTAs on the other SMs (HBM). The decode stream waits for the event
-        // that fires once every prefill CTA has begun, so the decode grid
-        // only takes the SMs left over: with both grids pending at once the
-        // hardware may place either first, and stream priority alone does
-        // not settle it. Decode CTAs beyond the free SMs start on the SMs
-        // that the prefill leaves as its queue runs dry; the decode merge
-        // follows the decode grid on its stream, beside the prefill.
-        cudaStream_t s = static_cast<cudaStream_t>(stream);
-        FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
-        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
-        const bool green = pl->g_pre != nullptr;  // partitions enforced: no placement order to keep
-        int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
-        if (rc == FNPU_OK) {
-            FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, green ? pl->e_fork : pl->e_started, 0));
-            const int dctas = 3 * (green ? pl->dec_sms : pl->num_sms);
-            rc = pl->desc.kv_fp8 ? launch_decode_fp8(p, pl->s_dec, dctas) : launch_decode_tma(p, pl->s_dec, dctas);
-        }
-        FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
-        FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
-        FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_pre, 0));
-        FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
-        return rc;
+bool run_pointers_ok(const fnpu_plan *pl, const void *q, const void *k_cache, const void *v_cache, const void *out,
+                     const float *lse) {
+    const bool latent = pl->desc.v_in_k_latent != 0;
+    if (!q || !k_cache || !out || !lse || (!latent && !v_cache)) return false;
+    const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_cache) |
+                          reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(lse) |
+                          (latent ? 0 : reinterpret_cast<uintptr_t>(v_cache));
+    return (mis & 15u) == 0;
+}
+
+// The decode kernel of a plan and its merge, on `stream`.
+int launch_decode(const fnpu_plan *pl, const AttnParams &p, void *stream, int ctas) {
+    return pl->desc.kv_fp8 ? launch_decode_fp8(p, stream, ctas) : launch_decode_tma(p, stream, ctas);
+}
+
+// Both phases side by side: pre_ctas persistent prefill CTAs (one per SM, the
+// tensor pipe; a decode CTA does not fit beside one) and decode CTAs on the
+// other SMs (HBM). The decode stream waits for the event that fires once
+// every prefill CTA has begun, so the decode grid only takes the SMs left
+// over: with both grids pending at once the hardware may place either first,
+// and stream priority alone does not settle it. Decode CTAs beyond the free
+// SMs start on the SMs that the prefill leaves as its queue runs dry; the
+// decode merge follows the decode grid on its stream, beside the prefill.
+int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
+    FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
+    const bool green = pl->g_pre != nullptr;  // partitions enforced: no placement order to keep
+    int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
+    if (rc == FNPU_OK) {
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, green ? pl->e_fork : pl->e_started, 0));
+        rc = launch_decode(pl, p, pl->s_dec, 3 * (green ? pl->dec_sms : pl->num_sms));
     }
+    FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
+    FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
+    FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_pre, 0));
+    FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
+    return rc;
+}
+
+}  // namespace
+}  // namespace fnpu
+
+extern "C" {
+
+int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache, const void *v_cache,
+                        void *out, float *lse, void *stream) {
+    if (!pl) return FNPU_EINVAL;
+    if (pl->num_tokens == 0) return FNPU_OK;
+    if (!run_pointers_ok(pl, q, k_cache, v_cache, out, lse)) return FNPU_EINVAL;
+    const AttnParams p = run_params(pl, q, k_cache, v_cache, out, lse);
+    if (pl->use_mla) return pl->use_mla_tc ? launch_mla_tc(p, stream) : launch_mla(p, stream);
+    if (pl->coloc) return run_colocated(pl, p, stream);
     int rc = pl->desc.kv_fp8 ? launch_decode_fp8(p, stream, 3 * pl->num_sms)
              : pl->use_dt    ? launch_decode_tma(p, stream, 3 * pl->num_sms)
                              : launch_decode_mma(p, stream);
@@ -1192,6 +1252,15 @@ int fnpu_plan_info(const fnpu_plan *pl, int32_t *prefill_items, int32_t *decode_
         *launches_per_run = (pl->num_pitems > 0) + (pl->num_ditems > 0) + (pl->num_mitems > 0) + (pl->num_mgroups > 0) +
                             (pl->num_jobs > 0 ? 1 : 0);  // FP8 staging: blocks and queries to f16
     if (workspace_bytes) *workspace_bytes = static_cast<int64_t>(pl->ws_cap);
+    return FNPU_OK;
+}
+
+// The decode share of a co-located plan, as a rounded percent of the SMs.
+int fnpu_plan_decode_share(const fnpu_plan *pl, int32_t *share_pct) {
+    if (!pl || !share_pct) return FNPU_EINVAL;
+    if (!pl->coloc || pl->num_sms <= 0) return FNPU_EUNSUPPORTED;
+    const int32_t k = pl->num_sms - pl->pre_ctas;
+    *share_pct = std::max<int32_t>(1, (200 * k + pl->num_sms) / (2 * pl->num_sms));  // rounded percent
     return FNPU_OK;
 }
 

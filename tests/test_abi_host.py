@@ -122,6 +122,8 @@ def test_append_and_run_reject_null_pointers():
     assert lib.fnpu_mixed_attn_run(None, None, None, None, None, None, None) == fnpu.FNPU_EINVAL
     assert lib.fnpu_plan_check(None, None) == fnpu.FNPU_EINVAL
     assert lib.fnpu_mixed_attn_replan(None, 0, None, None, None, None, 1, None, None) == fnpu.FNPU_EINVAL
+    share = ctypes.c_int32(-1)
+    assert lib.fnpu_plan_decode_share(None, ctypes.byref(share)) == fnpu.FNPU_EINVAL and share.value == -1
     lib.fnpu_plan_destroy(None)  # ignored
 
 

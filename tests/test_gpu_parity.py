@@ -583,3 +583,22 @@ def test_replan_rejects_bad_metadata_and_keeps_the_plan():
     st.attend()
     assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
     _compare(batch, *st.results())
+
+
+def test_planner_decode_share_is_reported():
+    """A co-located plan reports the decode share it uses: the one it was given
+    (to the rounding of SMs), or the planner's own choice, inside the
+    controller's range; a plan with one phase has none."""
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    st = DeviceStep(W.make_batch("qwen_coloc", seed=0), opts=fnpu.PlanOpts(0, 20, 0, 0))
+    assert abs(fnpu.plan_decode_share(st.plan) - 20) <= 1
+    st.replan(fnpu.PlanOpts(0, 0, 0, 0))
+    assert 1 <= fnpu.plan_decode_share(st.plan) <= 50
+    st.run()
+    out, lse = st.results()
+    _compare(st.batch, out, lse, tokens=_sample_tokens(st.batch, per_seq_rows=4))
+    one = DeviceStep(W.make_batch("qwen_prefill", seed=0))
+    with pytest.raises(fnpu.FnpuError) as e:
+        fnpu.plan_decode_share(one.plan)
+    assert e.value.code == fnpu.FNPU_EUNSUPPORTED

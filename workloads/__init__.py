@@ -339,6 +339,18 @@ def pairs(batch: Batch) -> int:
     return int((q * p + q * (q + 1) // 2).sum())
 
 
+def prefill_path_flops(batch: Batch) -> int:
+    """FLOPs of the rows that take the prefill path (sequences with more than
+    one query token: chunks and multi-token decodes): 2*Hq*pairs*(d_qk + d_v)
+    over those sequences only."""
+    sh = batch.shape
+    q = batch.query_len.astype(np.int64)
+    p = batch.context_len.astype(np.int64) - q
+    sel = q > 1
+    pr = int((q[sel] * p[sel] + q[sel] * (q[sel] + 1) // 2).sum())
+    return int(2 * sh.num_q_heads * pr * (sh.head_dim_qk + sh.head_dim_v))
+
+
 def algorithmic_work(batch: Batch, kv_fp8: bool = False) -> dict:
     """Algorithmic FLOPs and HBM bytes of one step (append + attention).
 
