@@ -192,12 +192,11 @@ std::vector<int32_t> cost_histogram(const std::vector<int64_t> &costs);
 // ties (more decode done while the prefill lasts).
 int32_t choose_decode_sms(const std::vector<int64_t> &item_tiles, double tile_scale, int64_t dec_bytes,
                           int32_t sms) {
-    int32_t best_k = 1;
-    double best_t = -1.0;
     const std::vector<int32_t> hist = cost_histogram(item_tiles);
     const double unit = tile_scale * kTileSec;  // seconds per cost unit
     std::vector<int32_t> loads;
-    for (int32_t k = 1; k <= sms / 2; ++k) {
+    // (prefill end, decode end) with k decode SMs
+    auto phases = [&](int32_t k) {
         const double tp = static_cast<double>(lpt_makespan(hist, sms - k, INT64_MAX, &loads)) * unit;
         double left = static_cast<double>(dec_bytes), t = 0.0;
         int32_t n = k;
@@ -213,7 +212,25 @@ int32_t choose_decode_sms(const std::vector<int64_t> &item_tiles, double tile_sc
             }
             if (ld < loads.size()) n += loads[ld];
         }
-        const double step = std::max(tp, t);
+        return std::make_pair(tp, t);
+    };
+    // The prefill end grows with k and the decode end shrinks, so the step
+    // max(Tp, Td) is shortest near the smallest k whose decode ends within
+    // the prefill: found by bisection, then the k around it are compared
+    // (the LPT makespan is not strictly monotone in the number of workers)
+    const int32_t kmax = std::max<int32_t>(sms / 2, 1);
+    int32_t lo = 1, hi = kmax;
+    while (lo < hi) {
+        const int32_t mid = (lo + hi) / 2;
+        const auto ph = phases(mid);
+        if (ph.second <= ph.first) hi = mid;
+        else lo = mid + 1;
+    }
+    int32_t best_k = 1;
+    double best_t = -1.0;
+    for (int32_t k = std::max<int32_t>(1, lo - 4); k <= std::min<int32_t>(kmax, lo + 4); ++k) {
+        const auto ph = phases(k);
+        const double step = std::max(ph.first, ph.second);
         if (best_t < 0 || step <= best_t) {
             best_t = step;
             best_k = k;
@@ -347,9 +364,25 @@ std::vector<int32_t> choose_prefill_splits(const std::vector<TcUnit> &units, int
         while (n > 1 && split_bound(units[i].ntiles, n, n - 1) > units[i].max_start) --n;
         nmax[i] = n;
     }
+    // split_units[c]: units longer than c tiles that may split. Under a cap
+    // of c exactly these split, each into two pieces or more, and a unit cut
+    // into n >= 2 pieces costs at least kTcItemCost + 2 kTcMergeCost more than
+    // whole; with the total of the unsplit items that bounds a candidate's
+    // total from below before its splits are worked out
+    std::vector<int32_t> split_units(static_cast<size_t>(maxc) + 2, 0);
+    for (size_t i = 0; i < units.size(); ++i)
+        if (nmax[i] >= 2) ++split_units[static_cast<size_t>(units[i].ntiles) - 1];
+    for (int64_t c = maxc - 1; c >= 0; --c) split_units[static_cast<size_t>(c)] += split_units[static_cast<size_t>(c) + 1];
+    const int64_t whole = total + static_cast<int64_t>(units.size()) * kTcItemCost;
     std::vector<int32_t> prev;
     for (int64_t cap : caps) {
         if (cap < 4) continue;
+        if (best_span >= 0) {
+            const int64_t nsplit = cap >= maxc ? 0 : split_units[static_cast<size_t>(cap)];
+            if (nsplit == 0) continue;  // no unit splits: the first candidate's items
+            const int64_t lb = whole + nsplit * (kTcItemCost + 2 * kTcMergeCost);
+            if ((lb + sms - 1) / sms >= best_span) continue;
+        }
         // ceil(ntiles / cap) = floor((ntiles - 1) / cap) + 1 in double, exact
         // for tile counts (below 2^26): a quotient that is not an integer has a
         // fraction of at least 1 / cap, above 1e-8, and the product errs by far
@@ -626,12 +659,20 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
                                       desc->num_q_heads / desc->num_kv_heads);
 
     const int32_t G = desc->num_q_heads / desc->num_kv_heads;
-    std::vector<SeqInfo> seqs(num_seqs);
-    std::vector<DecodeItem> ditems;
-    std::vector<PrefillItem> pitems;
-    std::vector<std::pair<int64_t, int32_t>> pcost;  // (cost, index) for LPT order
-    std::vector<TcUnit> tc_units;
-    std::vector<MergeGroup> mgroups;
+    // working lists, kept per thread across plans so that a re-plan
+    // allocates nothing once they have grown to the step's size
+    thread_local std::vector<SeqInfo> seqs;
+    thread_local std::vector<DecodeItem> ditems;
+    thread_local std::vector<PrefillItem> pitems;
+    thread_local std::vector<std::pair<int64_t, int32_t>> pcost;  // (cost, index) for LPT order
+    thread_local std::vector<TcUnit> tc_units;
+    thread_local std::vector<MergeGroup> mgroups;
+    seqs.assign(static_cast<size_t>(num_seqs), SeqInfo{});
+    ditems.clear();
+    pitems.clear();
+    pcost.clear();
+    tc_units.clear();
+    mgroups.clear();
 
     // decode split length: a TMA decode item streams every kv head of its
     // keys, and about two equal items per SM already keep HBM saturated, while
@@ -664,7 +705,8 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     // latent attention: every query row (prefill or decode) is 64-head blocks
     // over its visible keys, split into pieces of at most mla_split keys so
     // that about three CTAs per SM share the work; longest first
-    std::vector<MlaItem> mitems;
+    thread_local std::vector<MlaItem> mitems;
+    mitems.clear();
     int32_t mla_split = 0;
     int32_t mla_split_tiles = 0;
     if (pl->use_mla_tc) {
@@ -882,21 +924,17 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
         pl->num_tblocks = std::max(pl->num_jobs, 1);
     }
 
-    // longest prefill tiles first; decode items longest first as well
-    std::vector<PrefillItem> pordered(pitems.size());
+    // longest prefill tiles first; decode items longest first as well (the
+    // items are gathered in these orders straight into the upload below)
+    std::vector<int32_t> porder, dorder;
     {
-        std::vector<int64_t> cost(pitems.size());
+        thread_local std::vector<int64_t> cost;
+        cost.assign(pitems.size(), 0);
         for (const auto &pc : pcost) cost[static_cast<size_t>(pc.second)] = pc.first;
-        const std::vector<int32_t> order = longest_first(cost);
-        for (size_t i = 0; i < order.size(); ++i) pordered[i] = pitems[static_cast<size_t>(order[i])];
-    }
-    {
-        std::vector<int64_t> cost(ditems.size());
+        porder = longest_first(cost);
+        cost.resize(ditems.size());
         for (size_t i = 0; i < ditems.size(); ++i) cost[i] = ditems[i].key_end - ditems[i].key_begin;
-        const std::vector<int32_t> order = longest_first(cost);
-        std::vector<DecodeItem> sorted(ditems.size());
-        for (size_t i = 0; i < order.size(); ++i) sorted[i] = ditems[static_cast<size_t>(order[i])];
-        ditems.swap(sorted);
+        dorder = longest_first(cost);
     }
 
     std::stable_sort(mitems.begin(), mitems.end(), [](const MlaItem &a, const MlaItem &b) {
@@ -905,7 +943,7 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     pl->num_mitems = static_cast<int32_t>(mitems.size());
     pl->num_mgroups = static_cast<int32_t>(mgroups.size());
     pl->num_ditems = static_cast<int32_t>(ditems.size());
-    pl->num_pitems = static_cast<int32_t>(pordered.size());
+    pl->num_pitems = static_cast<int32_t>(pitems.size());
     pl->num_groups = groups;
     pl->num_parts = parts;
     pl->num_pparts = pparts;
@@ -936,7 +974,7 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     const size_t o_di = off; off = align_up(off + sizeof(DecodeItem) * std::max<size_t>(ditems.size(), 1), 256);
     const size_t o_mi = off; off = align_up(off + sizeof(MlaItem) * std::max<size_t>(mitems.size(), 1), 256);
     const size_t o_mg = off; off = align_up(off + sizeof(MergeGroup) * std::max<size_t>(mgroups.size(), 1), 256);
-    const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pordered.size(), 1), 256);
+    const size_t o_pi = off; off = align_up(off + sizeof(PrefillItem) * std::max<size_t>(pitems.size(), 1), 256);
     const size_t o_cnt = off; off = align_up(off + sizeof(int32_t) * std::max(groups, 1), 256);
     const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
     const size_t o_jobs = off; off = align_up(off + sizeof(Fp8StageJob) * std::max<size_t>(jobs.size(), 1), 256);
@@ -1018,12 +1056,18 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
         memcpy(h + o_bt + sizeof(int32_t) * static_cast<size_t>(s) * width,
                block_table + static_cast<int64_t>(s) * block_table_stride,
                sizeof(int32_t) * static_cast<size_t>((context_len[s] + bs - 1) / bs));
-    if (!ditems.empty()) memcpy(h + o_di, ditems.data(), sizeof(DecodeItem) * ditems.size());
+    {
+        DecodeItem *dst = reinterpret_cast<DecodeItem *>(h + o_di);
+        for (size_t i = 0; i < dorder.size(); ++i) dst[i] = ditems[static_cast<size_t>(dorder[i])];
+    }
     if (!mitems.empty()) memcpy(h + o_mi, mitems.data(), sizeof(MlaItem) * mitems.size());
     if (!mgroups.empty()) memcpy(h + o_mg, mgroups.data(), sizeof(MergeGroup) * mgroups.size());
     if (!jobs.empty()) memcpy(h + o_jobs, jobs.data(), sizeof(Fp8StageJob) * jobs.size());
     if (!tbt.empty()) memcpy(h + o_tbt, tbt.data(), sizeof(int32_t) * tbt.size());
-    if (!pordered.empty()) memcpy(h + o_pi, pordered.data(), sizeof(PrefillItem) * pordered.size());
+    {
+        PrefillItem *dst = reinterpret_cast<PrefillItem *>(h + o_pi);
+        for (size_t i = 0; i < porder.size(); ++i) dst[i] = pitems[static_cast<size_t>(porder[i])];
+    }
 
     uint8_t *d = static_cast<uint8_t *>(pl->d_ws);
     pl->d_seqs = reinterpret_cast<SeqInfo *>(d + o_seqs);
