@@ -491,8 +491,12 @@ namespace fnpu {
 namespace {
 // The tcgen05 prefill launch; over the FP8 cache, first the f16 staging of
 // the prefill sequences' blocks and of the queries, and the prefill reads those.
-int launch_prefill(const fnpu_plan *pl, const AttnParams &p, void *stream, int ctas, void *started) {
-    if (!pl->desc.kv_fp8) return launch_prefill_tc(p, stream, ctas, started);
+// A bf16 prefill launched on the stream of the kernel before it (pdl) is a
+// programmatic dependent launch: its CTAs set up while that kernel drains,
+// and its loaders wait for it before the first read.
+int launch_prefill(const fnpu_plan *pl, const AttnParams &p, void *stream, int ctas, void *started,
+                   bool pdl = false) {
+    if (!pl->desc.kv_fp8) return launch_prefill_tc(p, stream, ctas, started, false, pdl);
     const int rc = launch_fp8_stage(p.k_cache, p.v_cache, pl->d_jobs, pl->num_jobs, pl->d_tk, pl->d_tv, p.q, pl->d_tq,
                                     p.num_tokens * p.num_q_heads * p.head_dim_qk, stream);
     if (rc != FNPU_OK) return rc;
@@ -1223,9 +1227,26 @@ int launch_decode(const fnpu_plan *pl, const AttnParams &p, void *stream, int ct
 // decode merge follows the decode grid on its stream, beside the prefill.
 int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
-    FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
     const bool green = pl->g_pre != nullptr;  // partitions enforced: no placement order to keep
+    FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
+    if (!green && !pl->desc.kv_fp8) {
+        // The prefill grid goes on the caller's stream as a programmatic
+        // dependent of the kernel before it (the step's append): its CTAs take
+        // their SMs and set up while that kernel drains. The decode stream
+        // waits for the fork (everything before the prefill is done) and for
+        // the prefill grid's launch-completion event, as below.
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
+        int rc = launch_prefill(pl, p, s, pl->pre_ctas, pl->e_started, true);
+        if (rc == FNPU_OK) {
+            FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_started, 0));
+            rc = launch_decode(pl, p, pl->s_dec, 3 * pl->num_sms);
+        }
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, s));
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
+        return rc;
+    }
+    FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
     int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
     if (rc == FNPU_OK) {
         FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, green ? pl->e_fork : pl->e_started, 0));
@@ -1255,7 +1276,7 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
              : pl->use_dt    ? launch_decode_tma(p, stream, 3 * pl->num_sms)
                              : launch_decode_mma(p, stream);
     if (rc != FNPU_OK) return rc;
-    if (pl->use_tc) return launch_prefill(pl, p, stream, pl->num_sms, nullptr);
+    if (pl->use_tc) return launch_prefill(pl, p, stream, pl->num_sms, nullptr, true);
     return pl->desc.kv_fp8 ? launch_prefill_fp8(p, stream) : launch_prefill_mma(p, stream);
 }
 

@@ -161,8 +161,10 @@ int launch_split_merge(const AttnParams &p, void *stream);
 bool mla_supported(int d_qk, int d_v, int hq, int hkv);
 int mla_heads_per_item();
 // started (a cudaEvent_t, may be null): recorded once every CTA has begun;
-// f16: Q, K and V are f16 (d = 128 only), else bf16
-int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started = nullptr, bool f16 = false);
+// f16: Q, K and V are f16 (d = 128 only), else bf16; pdl: a programmatic
+// dependent launch of the kernel before it on `stream`
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started = nullptr, bool f16 = false,
+                      bool pdl = false);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);
 int prefill_tc_rows_per_item(int group);
 int prefill_tc_keys_per_tile();

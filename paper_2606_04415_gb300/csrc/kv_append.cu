@@ -24,6 +24,7 @@ __global__ void __launch_bounds__(256) kv_append_kernel(
     const uint4 *__restrict__ k_new, const uint4 *__restrict__ v_new,
     const int64_t *__restrict__ slots, int32_t num_tokens, int32_t k_chunks, int32_t v_chunks,
     uint4 *__restrict__ k_cache, uint4 *__restrict__ v_cache, int64_t num_slots) {
+    pdl_trigger();  // a dependent launch after this one may start its set-up now
     const int32_t per_tok = k_chunks + v_chunks;
     const int64_t total = static_cast<int64_t>(num_tokens) * per_tok;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;

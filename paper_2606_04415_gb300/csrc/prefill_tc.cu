@@ -39,6 +39,10 @@
 // columns); O0 at 256, O1 at 384.
 // Every mbarrier wait is bounded; a timeout raises the plan's error flag and
 // the CTA drains its tensor-core work, frees its tensor memory and exits.
+// Launched as a programmatic dependent of the kernel before it (the step's
+// KV append), the grid sets up while that kernel drains; the two loader
+// warps wait for it (griddepcontrol.wait) before their first read, and every
+// other warp reads global memory only after them.
 #include <math.h>
 
 #include "common.cuh"
@@ -197,6 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp >= 8) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsHelper));
     if (warp == 8 || warp == 9) {
+        pdl_wait();  // the cache writes of the kernel before (the step's append)
         // ---------------------------------- producers (8: scheduler, Q, K; 9: V)
         const bool is_k = warp == 8;
         if (lane == 0) {
@@ -678,7 +683,7 @@ bool encode_q_map(CUtensorMap *m, const void *base, int d, int hq, int64_t T, in
 }
 
 template <int DQ, int DV, bool F16>
-int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t started) {
+int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t started, bool pdl) {
     using Cfg = TcCfg<DQ, DV>;
     TcMaps maps;
     if (!encode_cache_map(&maps.k, p.k_cache, DQ, p.num_kv_heads, p.block_size, p.num_blocks, F16) ||
@@ -690,7 +695,7 @@ int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t st
     FNPU_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                                        cudaSharedmemCarveoutMaxShared));
     const int grid = p.num_pitems < max_ctas ? p.num_pitems : max_ctas;
-    FNPU_CUDA_TRY(launch_ex(kernel, grid, kThreads, Cfg::kSmemBytes, st, false, started, p, maps));
+    FNPU_CUDA_TRY(launch_ex(kernel, grid, kThreads, Cfg::kSmemBytes, st, pdl, started, p, maps));
     return FNPU_OK;
 }
 
@@ -709,18 +714,18 @@ int prefill_tc_rows_per_item(int group) { return 2 * (kRows / group); }
 // keys per K/V tile (the unit of the planner's key splits)
 int prefill_tc_keys_per_tile() { return kKeys; }
 
-int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started, bool f16) {
+int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started, bool f16, bool pdl) {
     if (p.num_pitems == 0) return FNPU_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaEvent_t ev = static_cast<cudaEvent_t>(started);
     if (f16)
-        return p.head_dim_qk == 128 && p.head_dim_v == 128 ? launch_tc<128, 128, true>(p, st, max_ctas, ev)
+        return p.head_dim_qk == 128 && p.head_dim_v == 128 ? launch_tc<128, 128, true>(p, st, max_ctas, ev, pdl)
                                                             : FNPU_EUNSUPPORTED;
-    if (p.head_dim_qk == 64 && p.head_dim_v == 64) return launch_tc<64, 64, false>(p, st, max_ctas, ev);
+    if (p.head_dim_qk == 64 && p.head_dim_v == 64) return launch_tc<64, 64, false>(p, st, max_ctas, ev, pdl);
     if (p.head_dim_qk == 128 && p.head_dim_v == 128)
-        return launch_tc<128, 128, false>(p, st, max_ctas, ev);
+        return launch_tc<128, 128, false>(p, st, max_ctas, ev, pdl);
     if (p.head_dim_qk == 192 && p.head_dim_v == 128)
-        return launch_tc<192, 128, false>(p, st, max_ctas, ev);
+        return launch_tc<192, 128, false>(p, st, max_ctas, ev, pdl);
     return FNPU_EUNSUPPORTED;
 }
 
