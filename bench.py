@@ -743,6 +743,9 @@ def run_fnpu(args):
                                "sustained": step_roof_sus / (step_ms * 1e-3),
                                "denominator": "max(F/bf16 peak, B/HBM peak) of measured"},
         "kernel_ms": {"append": sum(t_append) / K, "attention": attn_ms,
+                      "step_median": statistics.median(a + b for a, b in zip(t_append, t_attn)),
+                      "step_min": min(a + b for a, b in zip(t_append, t_attn)),
+                      "step_max": max(a + b for a, b in zip(t_append, t_attn)),
                       "prefill_phase": (sum(x[0] for x in phase) / len(phase)) if phase else None,
                       "decode_phase": (sum(x[1] for x in phase) / len(phase)) if phase else None},
         "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,

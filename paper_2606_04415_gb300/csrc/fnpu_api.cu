@@ -491,9 +491,9 @@ namespace fnpu {
 namespace {
 // The tcgen05 prefill launch; over the FP8 cache, first the f16 staging of
 // the prefill sequences' blocks and of the queries, and the prefill reads those.
-// A bf16 prefill launched on the stream of the kernel before it (pdl) is a
-// programmatic dependent launch: its CTAs set up while that kernel drains,
-// and its loaders wait for it before the first read.
+// With pdl a bf16 prefill grid is a programmatic dependent launch of the
+// kernel before it on `stream` (the step's append): its CTAs set up while that
+// kernel drains, and its loaders wait for it before the first read.
 int launch_prefill(const fnpu_plan *pl, const AttnParams &p, void *stream, int ctas, void *started,
                    bool pdl = false) {
     if (!pl->desc.kv_fp8) return launch_prefill_tc(p, stream, ctas, started, false, pdl);
@@ -1234,7 +1234,10 @@ int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
         // dependent of the kernel before it (the step's append): its CTAs take
         // their SMs and set up while that kernel drains. The decode stream
         // waits for the fork (everything before the prefill is done) and for
-        // the prefill grid's launch-completion event, as below.
+        // the prefill grid's launch-completion event. (Over the FP8 cache the
+        // staging kernel comes before the prefill; as its dependent the
+        // prefill's launch-completion event held the decode back by some 65 us,
+        // so that plan forks both phases as green contexts do, below.)
         FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
         int rc = launch_prefill(pl, p, s, pl->pre_ctas, pl->e_started, true);
         if (rc == FNPU_OK) {
@@ -1246,6 +1249,8 @@ int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
         FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
         return rc;
     }
+    // green contexts (each phase on its partition's stream, both from the
+    // fork) and the FP8 cache (the decode after the prefill grid's start)
     FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
     int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
     if (rc == FNPU_OK) {
