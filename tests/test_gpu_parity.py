@@ -602,3 +602,36 @@ def test_planner_decode_share_is_reported():
     with pytest.raises(fnpu.FnpuError) as e:
         fnpu.plan_decode_share(one.plan)
     assert e.value.code == fnpu.FNPU_EUNSUPPORTED
+
+
+@pytest.mark.parametrize("what", ["q", "cache"])
+def test_prefill_waits_for_the_kernel_before_it(what):
+    """The tcgen05 prefill grid is a programmatic dependent launch of the kernel
+    before it on the stream. Here that kernel is not the library's append but a
+    copy that writes the queries (or the whole cache) the step then reads,
+    replacing NaN: every output must still match the oracle, so the prefill's
+    loaders waited for the copy to finish."""
+    batch = _coloc_small_batch()
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    st = DeviceStep(batch)
+    st.append()
+    torch.cuda.synchronize()
+    dst = st.q if what == "q" else st.k_cache
+    good = dst.clone()
+    dst.fill_(float("nan"))
+    torch.cuda.synchronize()
+    dst.copy_(good)  # the kernel just before the attention on the same stream
+    st.attend()
+    out, lse = st.results()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK
+    _compare(batch, out, lse)
+
+
+def _coloc_small_batch():
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(21)
+    ql = [400, 1, 1, 129, 1] + [1] * 12
+    ctx = [400 + 1700, 700, 1500, 129 + 40, 33] + list(rng.integers(20, 3000, size=12))
+    ph = [0, 1, 1, 0, 1] + [1] * 12
+    return W.build_batch(sh, ql, ctx, ph, rng, name="coloc_pdl")
