@@ -1229,17 +1229,18 @@ int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bool green = pl->g_pre != nullptr;  // partitions enforced: no placement order to keep
     FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
-    if (!green && !pl->desc.kv_fp8) {
-        // The prefill grid goes on the caller's stream as a programmatic
-        // dependent of the kernel before it (the step's append): its CTAs take
-        // their SMs and set up while that kernel drains. The decode stream
-        // waits for the fork (everything before the prefill is done) and for
-        // the prefill grid's launch-completion event. (Over the FP8 cache the
-        // staging kernel comes before the prefill; as its dependent the
-        // prefill's launch-completion event held the decode back by some 65 us,
-        // so that plan forks both phases as green contexts do, below.)
+    if (!green) {
+        // The prefill grid goes on the caller's stream (a fork to a library
+        // stream costs the wait across streams before it starts), as a
+        // programmatic dependent of the kernel before it (the step's append):
+        // its CTAs take their SMs and set up while that kernel drains. The
+        // decode stream waits for the fork (everything before the prefill is
+        // done) and for the prefill grid's launch-completion event. (Over the
+        // FP8 cache the staging kernel comes before the prefill, which is then
+        // an ordinary launch: as the staging's dependent, the prefill's
+        // launch-completion event held the decode back by some 65 us.)
         FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
-        int rc = launch_prefill(pl, p, s, pl->pre_ctas, pl->e_started, true);
+        int rc = launch_prefill(pl, p, s, pl->pre_ctas, pl->e_started, !pl->desc.kv_fp8);
         if (rc == FNPU_OK) {
             FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_started, 0));
             rc = launch_decode(pl, p, pl->s_dec, 3 * pl->num_sms);
@@ -1249,13 +1250,12 @@ int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
         FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
         return rc;
     }
-    // green contexts (each phase on its partition's stream, both from the
-    // fork) and the FP8 cache (the decode after the prefill grid's start)
+    // green contexts: each phase on its partition's stream, both from the fork
     FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_pre, pl->e_fork, 0));
-    int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, green ? nullptr : pl->e_started);
+    int rc = launch_prefill(pl, p, pl->s_pre, pl->pre_ctas, nullptr);
     if (rc == FNPU_OK) {
-        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, green ? pl->e_fork : pl->e_started, 0));
-        rc = launch_decode(pl, p, pl->s_dec, 3 * (green ? pl->dec_sms : pl->num_sms));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
+        rc = launch_decode(pl, p, pl->s_dec, 3 * pl->dec_sms);
     }
     FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, pl->s_pre));
     FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
