@@ -635,3 +635,31 @@ def _coloc_small_batch():
     ctx = [400 + 1700, 700, 1500, 129 + 40, 33] + list(rng.integers(20, 3000, size=12))
     ph = [0, 1, 1, 0, 1] + [1] * 12
     return W.build_batch(sh, ql, ctx, ph, rng, name="coloc_pdl")
+
+
+def test_prefill_chunk_on_a_very_long_prefix():
+    """A Qwen-shape chunk of 256 tokens on a 40000-token prefix (316 key tiles
+    per item), beside a few decodes: long tile loops, key splits across CTAs
+    and their merge at scale; sampled rows against the oracle."""
+    sh = W.SHAPES["qwen"]
+    rng = np.random.default_rng(404)
+    ql = [256, 1, 1, 1]
+    ctx = [40000 + 256, 3000, 17, 40001]
+    ph = [0, 1, 1, 1]
+    batch = W.build_batch(sh, ql, ctx, ph, rng, name="long_prefix")
+    st = _step(batch)
+    out, lse = st.results()
+    qs = batch.query_start
+    toks = np.asarray(sorted({int(qs[0]) + r for r in (0, 1, 35, 36, 127, 200, 255)} | {int(qs[s]) for s in (1, 2, 3)}),
+                      np.int64)
+    _compare(batch, out, lse, tokens=toks)
+
+
+@pytest.mark.parametrize("seed", [1, 3, 7])
+def test_qwen_coloc_other_seeds_sampled_rows(seed):
+    """The co-located Qwen workload at other prefix draws (shorter and longer
+    prefixes, other decode shares chosen by the planner): sampled rows."""
+    batch = W.make_batch("qwen_coloc", seed=seed)
+    st = _step(batch)
+    out, lse = st.results()
+    _compare(batch, out, lse, tokens=_sample_tokens(batch, per_seq_rows=6, seed=seed))
