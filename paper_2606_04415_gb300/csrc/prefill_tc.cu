@@ -34,7 +34,9 @@
 //                   issue order, so S_w(j+1) overwrites P_w(j) only after
 //                   PV_w(j) has read it, and when S_w(j) is complete so is
 //                   PV_w(j-1) -- the softmax may rescale O_w at that point
-//                   without a further wait.
+//                   without a further wait. With a single V stage (192-wide
+//                   keys) the order is PV_0(j), PV_1(j), S_0(j+1), S_1(j+1),
+//                   so that V(j+1) loads while both S of the next tile run.
 // TMEM (512 columns): S0 at 0, S1 at 128 (fp32, P over their first 64
 // columns); O0 at 256, O1 at 384.
 // Every mbarrier wait is bounded; a timeout raises the plan's error flag and
@@ -385,7 +387,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issue_pv(0, vst, j > 0 ? 1u : 0u);
                 if (j == n - 1) tc::commit_warp(ODONE(0));
                 const bool more = j + 1 < n;
-                if (more) {
+                // (one V stage: both P V first, so that the next V tile loads
+                // while both S of the next key tile run)
+                constexpr bool kPvFirst = Cfg::kVStages == 1;
+                if (!kPvFirst && more) {
                     if (!wait(KFULL(gk % kKStages), (gk / kKStages) & 1)) { ok = false; break; }
                     tc::fence_after_sync();
                     issue_s(0, gk % kKStages);
@@ -398,6 +403,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::commit_warp(VEMPTY(vst));
                 ++gv;
                 if (j == n - 1) tc::commit_warp(ODONE(1));
+                if (kPvFirst && more) {
+                    if (!wait(KFULL(gk % kKStages), (gk / kKStages) & 1)) { ok = false; break; }
+                    tc::fence_after_sync();
+                    issue_s(0, gk % kKStages);
+                }
                 if (more) {
                     issue_s(1, gk % kKStages);
                     tc::commit_warp(KEMPTY(gk % kKStages));
