@@ -54,6 +54,7 @@ NCU_TRAFFIC = {
     "qwen_coloc": 33.5e6,        # prefill_tc 33.3 MB read + 0.21 MB write
     "qwen_decode": 308.9e6,      # decode_tma 308.15 MB read + 0.7 MB write
     "qwen_decode_fp8": 159.6e6,  # decode_fp8 159.16 MB read + 0.4 MB write
+    "mla_prefill_expand": 203.4e6,  # prefill_tc<192, 128> 188.9 MB read + 14.5 MB write
 }
 
 
@@ -424,7 +425,7 @@ def run_fnpu_mla_expand(args):
     roof = {"bound": "tensor", "achieved": F_attn / (t_att * 1e-3) / 1e12, "peak": peaks["bf16_tflops"],
             "unit": "TFLOP/s", "kernel": "prefill_tc_kernel<192, 128> (the attention call)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = args.traffic
+    roof["traffic"] = args.traffic if args.traffic is not None else NCU_TRAFFIC.get(args.workload + "_expand")
     roof["peak_source"] = peaks["source"] + " burst"
     T = batch.num_tokens
     line = {
