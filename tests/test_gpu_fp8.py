@@ -242,3 +242,35 @@ def test_fp8_colocated_in_green_context_partitions():
     _compare(batch, out, lse, kp, vp)
     pre, dec = fnpu.plan_phase_ms(st.plan)
     assert pre > 0 and dec > 0
+
+
+@pytest.mark.parametrize("case", range(10))
+def test_fp8_random_mixed_step_all_rows(case):
+    """Randomised mixes over the FP8 cache (Hkv = 4, d = 128, 16-slot blocks;
+    2 to 8 query heads per kv head): one-token and multi-token decodes,
+    chunks with and without a prefix, under random decode shares, key-split
+    lengths and launch modes. The pools must equal the reference's bit for
+    bit and every row must match the FP8 oracle."""
+    rng = np.random.default_rng(5000 + case)
+    hq = int(rng.choice([8, 12, 16, 28, 32]))
+    S = int(rng.integers(2, 11))
+    ql, ctx, ph = [], [], []
+    for _ in range(S):
+        kind = rng.choice(["decode", "decode", "multi", "chunk", "chunk_prefix"])
+        if kind == "decode":
+            ql.append(1), ctx.append(int(rng.integers(1, 3000))), ph.append(1)
+        elif kind == "multi":
+            q = int(rng.integers(2, 8))
+            ql.append(q), ctx.append(q + int(rng.integers(0, 2000))), ph.append(1)
+        elif kind == "chunk":
+            q = int(rng.integers(1, 300))
+            ql.append(q), ctx.append(q), ph.append(0)
+        else:
+            q = int(rng.integers(2, 300))
+            ql.append(q), ctx.append(q + int(rng.integers(1, 2500))), ph.append(0)
+    batch = _batch(ctx, hq=hq, seed=70 + case, ql=ql, phase=ph)
+    share = int(rng.choice([0, 0, 3, 20, 45]))
+    split = int(rng.choice([0, 0, 64, 256]))
+    flags = int(rng.choice([0, 0, 0, 1, 2]))  # separate launches / the mma.sync prefill
+    _, out, lse, kp, vp = _run(batch, seed=70 + case, split=split, flags=flags, share=share)
+    _compare(batch, out, lse, kp, vp)
