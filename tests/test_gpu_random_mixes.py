@@ -1,4 +1,5 @@
-"""Randomised mixed steps against the fp64 oracle, every query row.
+"""Randomised mixed steps against the fp64 oracle, every query row (GQA and
+absorbed latent attention).
 
 Each case draws a head shape (GQA groups 1 to 8, head widths 64 and 128,
 block sizes 16 to 64), a mix of sequences (one-token decodes, multi-token
@@ -79,5 +80,54 @@ def test_random_mixed_step_all_rows(case):
     assert eo <= O_TOL, f"case {case} (share {share}, split {split}, flags {flags}): max |dO| = {eo}"
     assert el <= LSE_TOL, f"case {case} (share {share}, split {split}, flags {flags}): max |dLSE| = {el}"
     st.attend()  # the cache already holds the step's rows; same plan, same bits
+    out2, lse2 = st.results()
+    assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
+
+
+def _draw_mla(case):
+    rng = np.random.default_rng(7000 + case)
+    bs = int(rng.choice([16, 32, 64]))
+    shape = W.Shape(128, 1, 576, 512, bs, True)
+    S = int(rng.integers(2, 7))
+    ql, ctx, ph = [], [], []
+    for _ in range(S):
+        kind = rng.choice(["decode", "decode", "multi", "chunk", "chunk_prefix"])
+        if kind == "decode":
+            ql.append(1), ctx.append(int(rng.integers(1, 4000))), ph.append(1)
+        elif kind == "multi":
+            q = int(rng.integers(2, 5))
+            ql.append(q), ctx.append(q + int(rng.integers(0, 1500))), ph.append(1)
+        elif kind == "chunk":
+            q = int(rng.integers(1, 64))
+            ql.append(q), ctx.append(q), ph.append(0)
+        else:
+            q = int(rng.integers(2, 64))
+            ql.append(q), ctx.append(q + int(rng.integers(1, 700))), ph.append(0)
+    batch = W.build_batch(shape, ql, ctx, ph, rng, name=f"random_mla_{case}")
+    return batch, int(rng.choice([0, 0, NO_TC]))
+
+
+@pytest.mark.parametrize("case", range(10))
+def test_random_latent_step_all_rows(case):
+    """Absorbed MLA (128 heads on one 576-wide latent row, V its first 512
+    columns) on random mixes: latent blocks of 16 to 64 slots, decodes long
+    enough to be cut into merged pieces, multi-token decodes and chunks; the
+    latent append bit-exact, every row against the oracle, and a second run
+    identical."""
+    import paper_2606_04415_gb300 as fnpu
+    from paper_2606_04415_gb300.step import DeviceStep
+    batch, flags = _draw_mla(case)
+    st = DeviceStep(batch, opts=fnpu.PlanOpts(0, 0, 0, flags))
+    st.run()
+    out, lse = st.results()
+    assert fnpu.plan_check(st.plan) == fnpu.FNPU_OK and fnpu.check() == fnpu.FNPU_OK
+    kc, _ = st.cache_bits()
+    assert np.array_equal(kc, oracle.kv_append(batch.k_cache, batch.k_new, batch.slot_mapping))
+    ref_o, ref_l, _, _ = oracle.run_step(batch)
+    assert np.isfinite(out).all() and np.isfinite(lse).all()
+    eo, el = np.abs(out - ref_o).max(), np.abs(lse - ref_l).max()
+    assert eo <= O_TOL, f"case {case} (flags {flags}): max |dO| = {eo}"
+    assert el <= LSE_TOL, f"case {case} (flags {flags}): max |dLSE| = {el}"
+    st.attend()
     out2, lse2 = st.results()
     assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
