@@ -495,8 +495,9 @@ def pipelined_e2e(st, host_in, host_out, steps, warmup, replan_opts=None):
     come down while step n - 1 computes; two device buffer sets alternate, with
     events ordering each set's reuse. With replan_opts, every step is also
     re-planned from its host metadata (fnpu_mixed_attn_replan) while the device
-    works on the step before. Returns ms per step: device time from the first
-    copy up to the last copy down, over `steps` steps (after `warmup`). No L2
+    works on the step before. Returns (ms per step of device time from the
+    first copy up to the last copy down, over `steps` steps after `warmup`;
+    ms per step the host took to issue them). No L2
     flush here: a step reads far more than L2 holds."""
     import torch
     comp = torch.cuda.current_stream()
@@ -521,6 +522,7 @@ def pipelined_e2e(st, host_in, host_out, steps, warmup, replan_opts=None):
             if i == warmup:
                 torch.cuda.synchronize()
                 t0.record(up)
+                h0 = time.perf_counter()
             with torch.cuda.stream(up):
                 if i >= 2:
                     up.wait_event(done[b])  # the set's previous step has read its inputs
@@ -545,12 +547,13 @@ def pipelined_e2e(st, host_in, host_out, steps, warmup, replan_opts=None):
                 hout[b][1].copy_(outs[b][1], non_blocking=True)
                 drained[b].record(down)
         t1.record(down)
+        host_ms = (time.perf_counter() - h0) * 1e3 / steps  # enqueueing only (no sync inside the loop)
         torch.cuda.synchronize()
     finally:
         for n in names:
             setattr(st, n, orig[n])
         st.out, st.lse = orig_out
-    return t0.elapsed_time(t1) / steps
+    return t0.elapsed_time(t1) / steps, host_ms
 
 
 def _fp8_workload_ok(batch):
@@ -742,9 +745,11 @@ def run_fnpu(args):
     e2e = e2e_by_mode["plan_once"]
     e2e_replan = e2e_by_mode["replan_every_step"]
     host_in = {"q": h_q, "k_new": h_k, "v_new": h_v, "slot_mapping": h_s}
-    e2e_pipe = max_over_ranks(pipelined_e2e(st, host_in, (h_o, h_l), K, args.warmup), ws, dev)
-    e2e_pipe_replan = max_over_ranks(pipelined_e2e(st, host_in, (h_o, h_l), K, args.warmup, replan_opts=share_opts),
-                                     ws, dev)
+    e2e_pipe, host_pipe = pipelined_e2e(st, host_in, (h_o, h_l), K, args.warmup)
+    e2e_pipe = max_over_ranks(e2e_pipe, ws, dev)
+    e2e_pipe_replan, host_pipe_replan = pipelined_e2e(st, host_in, (h_o, h_l), K, args.warmup,
+                                                      replan_opts=share_opts)
+    e2e_pipe_replan = max_over_ranks(e2e_pipe_replan, ws, dev)
 
     # roofline of the dominant kernel: for a co-located step the prefill
     # kernel (its tile FLOPs over the prefill phase of the step, from the fork
@@ -797,15 +802,23 @@ def run_fnpu(args):
                       "step_max": max(t_step),
                       "prefill_phase": (sum(x[0] for x in phase) / len(phase)) if phase else None,
                       "decode_phase": (sum(x[1] for x in phase) / len(phase)) if phase else None},
-        "e2e": {"value": job_throughput(ws, T, e2e), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e,
-                "serial": "each step's copies up, step, copies down, one after the other; L2 flushed between steps",
-                "replan_every_step": {"value": job_throughput(ws, T, e2e_replan), "ms_per_step": e2e_replan},
-                "pipelined": {"value": job_throughput(ws, T, e2e_pipe), "ms_per_step": e2e_pipe,
-                              "how": "step n's copies up and step n-1's copies down overlap step n-1's compute "
-                                     "(copy streams, two buffer sets); no L2 flush, a step reads > L2"},
-                "pipelined_replan_every_step": {"value": job_throughput(ws, T, e2e_pipe_replan),
-                                                "ms_per_step": e2e_pipe_replan}},
+        # end to end as a serving loop runs it: every step's inputs up from pinned
+        # host memory and its outputs down, on copy streams that overlap the
+        # step before; the same with the copies and the step one after the
+        # other below ("serial")
+        "e2e": {"value": job_throughput(ws, T, e2e_pipe), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_pipe,
+                "how": "pipelined: step n's copies up and step n-1's copies down overlap step n-1's compute "
+                       "(copy streams, two buffer sets), timed from the first copy up to the last copy down "
+                       "over the K steps; no L2 flush, a step reads > L2",
+                "host_ms_per_step": host_pipe,
+                "replan_every_step": {"value": job_throughput(ws, T, e2e_pipe_replan),
+                                      "ms_per_step": e2e_pipe_replan, "host_ms_per_step": host_pipe_replan},
+                "serial": {"value": job_throughput(ws, T, e2e), "ms_per_step": e2e,
+                           "how": "each step's copies up, step, copies down, one after the other; "
+                                  "L2 flushed between steps",
+                           "replan_every_step": {"value": job_throughput(ws, T, e2e_replan),
+                                                 "ms_per_step": e2e_replan}}},
         "gpu_launches": K * (1 + info["launches_per_run"]),  # the append and the run's launches
         "clocks": clk,
     }
