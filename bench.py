@@ -654,16 +654,15 @@ def run_fnpu(args):
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    # the timed steps: append (fnpu_kv_append) + attention (fnpu_mixed_attn_run),
-    # events only around the whole step (an event between the two calls sits
-    # between the append and the prefill grid that is its dependent launch,
-    # and costs the step about 2 us)
+    # the timed steps: fnpu_mixed_step (the append, then the attention), events
+    # only around the whole step (an event between the append and the
+    # attention sits between the append and the prefill grid that is its
+    # dependent launch, and costs the step about 2 us)
     with ClockSampler(local) as clocks:
         for i in range(K):
             _flush_l2(flush, flush_r)  # evict L2 between timed steps (outside the events)
             ev[i][0].record(stream)
-            st.append()
-            st.attend()
+            st.run()
             ev[i][1].record(stream)
         torch.cuda.synchronize(dev)
         if ws > 1:

@@ -12,6 +12,7 @@
  *                           work list -- the phase-aware dispatch of Sec. 3.4
  *   fnpu_mixed_attn_run     causal attention of every query over its sequence's
  *                           cached keys, one launch on the caller's stream
+ *   fnpu_mixed_step         the append and the attention of a step in one call
  *
  * As in the paper's control path (Sec. 3.2), calls pass metadata and pointers
  * only: tensors stay in device memory owned by the caller; the library never
@@ -114,6 +115,14 @@ typedef struct {
                                          over disjoint SM partitions (the decode share rounded
                                          up to the device's partition granularity); plan
                                          fails with FNPU_EUNSUPPORTED where they cannot be made */
+#define FNPU_PLAN_FUSED_APPEND 8      /* fnpu_mixed_step: where the prefill runs on the tcgen05
+                                         kernel over a bf16 cache (not in green contexts), its
+                                         CTAs write the prefill-path rows themselves and a small
+                                         kernel writes the decode rows, instead of one append
+                                         kernel ahead of the run. Results are the same bit for
+                                         bit; on the Qwen co-located and prefill-only steps it
+                                         measured slower than the default (the append kernel's
+                                         time is hidden by the prefill grid's dependent launch) */
 
 /*
  * KV append: for each token t in [0, num_tokens) with slot_mapping[t] >= 0,
@@ -200,6 +209,24 @@ int fnpu_mixed_attn_replan(fnpu_plan *plan, int32_t num_seqs, const int32_t *que
  */
 int fnpu_mixed_attn_run(const fnpu_plan *plan, const void *q, const void *k_cache,
                         const void *v_cache, void *out, float *lse, void *stream);
+
+/*
+ * A whole step: fnpu_kv_append of the step's new rows followed by
+ * fnpu_mixed_attn_run, with the same arguments and the same results bit for
+ * bit (the shared KV pool of both phases, Sec. 3.4). k_new, v_new and
+ * slot_mapping are as for fnpu_kv_append, with the plan's token count; their
+ * rows are the planned step's tokens in order. By default the two calls are
+ * made in turn. With FNPU_PLAN_FUSED_APPEND, where the plan's prefill runs on
+ * the tcgen05 kernel over a bf16 cache (and not in green contexts), that
+ * kernel's CTAs write the prefill-path rows themselves before they read the
+ * cache (a cooperative launch: they wait for one another, bounded), and a
+ * small kernel writes the decode rows ahead of the decode kernel. An
+ * out-of-range slot raises the library-wide flag (fnpu_check), as
+ * fnpu_kv_append does; a bounded wait that runs out raises the plan's flag.
+ * Errors: FNPU_EINVAL (NULL or misaligned pointers), FNPU_ECUDA.
+ */
+int fnpu_mixed_step(const fnpu_plan *plan, const void *k_new, const void *v_new, const int64_t *slot_mapping,
+                    const void *q, void *k_cache, void *v_cache, void *out, float *lse, void *stream);
 
 
 /* Synchronise `stream`, then read and clear the plan's device error flag:

@@ -36,13 +36,14 @@ FNPU_EDEVICE_RANGE = -6
 PLAN_SEPARATE_LAUNCHES = 1
 PLAN_NO_TCGEN05 = 2
 PLAN_GREEN_CONTEXTS = 4
+PLAN_FUSED_APPEND = 8
 
 EXPORTED = (
     "fnpu_kv_append", "fnpu_mixed_attn_plan", "fnpu_mixed_attn_plan_ex", "fnpu_mixed_attn_run",
     "fnpu_plan_check", "fnpu_check", "fnpu_plan_destroy", "fnpu_plan_info", "fnpu_status_str",
     "fnpu_version", "fnpu_decode_attn_noalloc", "fnpu_last_cuda_error", "fnpu_plan_phase_ms",
     "fnpu_dispatch_next_share", "fnpu_mla_expand", "fnpu_mixed_attn_replan",
-    "fnpu_plan_decode_share",
+    "fnpu_plan_decode_share", "fnpu_mixed_step",
 )
 
 
@@ -93,6 +94,7 @@ def load(build_if_missing: bool = True):
                                             ctypes.POINTER(PlanOpts), P, ctypes.POINTER(P)]
     lib.fnpu_mixed_attn_replan.argtypes = [P, i32, P, P, P, P, i32, ctypes.POINTER(PlanOpts), P]
     lib.fnpu_mixed_attn_run.argtypes = [P, P, P, P, P, P, P]
+    lib.fnpu_mixed_step.argtypes = [P, P, P, P, P, P, P, P, P, P]
     lib.fnpu_plan_decode_share.argtypes = [P, ctypes.POINTER(i32)]
     lib.fnpu_mla_expand.argtypes = [ctypes.POINTER(AttnDesc), P, P, i32, P, P, P, P, P, P]
     lib.fnpu_plan_check.argtypes = [P, P]
@@ -263,6 +265,16 @@ def mixed_attn_run(plan: Plan, q, k_cache, v_cache, out, lse, stream=None) -> No
                                     _dptr(out), _dptr(lse), _stream(stream))
     if rc != FNPU_OK:
         raise FnpuError(rc, "fnpu_mixed_attn_run")
+
+
+def mixed_step(plan: Plan, k_new, v_new, slot_mapping, q, k_cache, v_cache, out, lse, stream=None) -> None:
+    """Append of the step's new rows and attention of every planned query in
+    one call (``fnpu_mixed_step``; the same results as ``kv_append`` then
+    ``mixed_attn_run``)."""
+    rc = load().fnpu_mixed_step(plan.handle, _dptr(k_new), _dptr(v_new), _dptr(slot_mapping), _dptr(q),
+                                _dptr(k_cache), _dptr(v_cache), _dptr(out), _dptr(lse), _stream(stream))
+    if rc != FNPU_OK:
+        raise FnpuError(rc, "fnpu_mixed_step")
 
 
 def decode_attn_noalloc(desc: AttnDesc, context_len, block_table, max_context_len: int, q,

@@ -116,11 +116,18 @@ __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\
 // writes); `started`, if not null, is recorded once every CTA of this grid
 // has begun (a launch completion event; the runtime treats it as best
 // effort, and at worst it fires when the grid ends).
+// `cooperative` (launch_coop) guarantees that every CTA of the grid is
+// resident at once, which a grid whose CTAs wait for one another needs.
 template <typename... Args>
-cudaError_t launch_ex(void (*kernel)(Args...), int grid, int threads, size_t smem, cudaStream_t st, bool after_prev,
-                      cudaEvent_t started, const Args &...args) {
-    cudaLaunchAttribute attr[2];
+cudaError_t launch_coop(void (*kernel)(Args...), int grid, int threads, size_t smem, cudaStream_t st,
+                        bool after_prev, cudaEvent_t started, bool cooperative, const Args &...args) {
+    cudaLaunchAttribute attr[3];
     int n = 0;
+    if (cooperative) {
+        attr[n].id = cudaLaunchAttributeCooperative;
+        attr[n].val.cooperative = 1;
+        ++n;
+    }
     if (after_prev) {
         attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[n].val.programmaticStreamSerializationAllowed = 1;
@@ -140,6 +147,11 @@ cudaError_t launch_ex(void (*kernel)(Args...), int grid, int threads, size_t sme
     cfg.attrs = attr;
     cfg.numAttrs = n;
     return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+template <typename... Args>
+cudaError_t launch_ex(void (*kernel)(Args...), int grid, int threads, size_t smem, cudaStream_t st, bool after_prev,
+                      cudaEvent_t started, const Args &...args) {
+    return launch_coop(kernel, grid, threads, smem, st, after_prev, started, false, args...);
 }
 
 // One 32-byte global store (8 x 32 bits; the address is 32-byte aligned).

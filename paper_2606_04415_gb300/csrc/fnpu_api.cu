@@ -64,6 +64,10 @@ struct fnpu_plan {
     fnpu::PrefillItem *d_pitems = nullptr;
     int32_t *d_counters = nullptr;
     int32_t *d_err = nullptr;
+    // the step's tokens by queue (tcgen05 prefill plans): rows the prefill
+    // grid appends itself in fnpu_mixed_step, and the decode rows
+    int32_t *d_ftok = nullptr, *d_dtok = nullptr;
+    int32_t num_ftok = 0, num_dtok = 0;
     float *d_part_lse = nullptr;
     float *d_part_o = nullptr;
     int32_t *d_pcounters = nullptr;
@@ -952,6 +956,16 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     pl->num_parts = parts;
     pl->num_pparts = pparts;
     pl->num_pgroups = pgroups;
+    // the step's tokens by queue, for the append inside the prefill grid
+    thread_local std::vector<int32_t> ftok, dtok;
+    ftok.clear();
+    dtok.clear();
+    if ((o.flags & FNPU_PLAN_FUSED_APPEND) && pl->use_tc && !pl->use_mla && !pitems.empty()) {
+        for (int32_t s = 0; s < num_seqs; ++s)
+            for (int32_t i = 0; i < query_len[s]; ++i) (decode_queue(s) ? dtok : ftok).push_back(seqs[s].q_start + i);
+    }
+    pl->num_ftok = static_cast<int32_t>(ftok.size());
+    pl->num_dtok = static_cast<int32_t>(dtok.size());
     if (pl->coloc) {
         // made once per plan and kept across re-plans (green streams above)
         int lo = 0, hi = 0;
@@ -971,7 +985,8 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     // workspace: the error flag and work queues (kept across re-plans), the
     // metadata (uploaded), then scratch (never read before written)
     size_t off = 0;
-    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);  // err + work queues
+    // err [0], work queues [2..5], the count of the append inside the prefill grid [6]
+    const size_t o_err = off; off = align_up(off + sizeof(int32_t) * 8, 256);
     const size_t o_meta = off;
     const size_t o_seqs = off; off = align_up(off + sizeof(SeqInfo) * std::max(num_seqs, 1), 256);
     const size_t o_bt = off; off = align_up(off + sizeof(int32_t) * static_cast<size_t>(std::max(num_seqs, 1)) * width, 256);
@@ -983,6 +998,8 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     const size_t o_pcnt = off; off = align_up(off + sizeof(int32_t) * 8 * static_cast<size_t>(std::max(pgroups, 1)), 256);
     const size_t o_jobs = off; off = align_up(off + sizeof(Fp8StageJob) * std::max<size_t>(jobs.size(), 1), 256);
     const size_t o_tbt = off; off = align_up(off + sizeof(int32_t) * std::max<size_t>(tbt.size(), 1), 256);
+    const size_t o_ftok = off; off = align_up(off + sizeof(int32_t) * std::max<size_t>(ftok.size(), 1), 256);
+    const size_t o_dtok = off; off = align_up(off + sizeof(int32_t) * std::max<size_t>(dtok.size(), 1), 256);
     const size_t meta_bytes = off;
     // query heads per partial
     const int32_t part_rows = pl->use_mla_tc ? desc->num_q_heads
@@ -1068,6 +1085,8 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     if (!mgroups.empty()) memcpy(h + o_mg, mgroups.data(), sizeof(MergeGroup) * mgroups.size());
     if (!jobs.empty()) memcpy(h + o_jobs, jobs.data(), sizeof(Fp8StageJob) * jobs.size());
     if (!tbt.empty()) memcpy(h + o_tbt, tbt.data(), sizeof(int32_t) * tbt.size());
+    if (!ftok.empty()) memcpy(h + o_ftok, ftok.data(), sizeof(int32_t) * ftok.size());
+    if (!dtok.empty()) memcpy(h + o_dtok, dtok.data(), sizeof(int32_t) * dtok.size());
     {
         PrefillItem *dst = reinterpret_cast<PrefillItem *>(h + o_pi);
         for (size_t i = 0; i < porder.size(); ++i) dst[i] = pitems[static_cast<size_t>(porder[i])];
@@ -1089,6 +1108,8 @@ int plan_fill(fnpu_plan *pl, const fnpu_attn_desc *desc, int32_t num_seqs, const
     pl->d_ppart_o = reinterpret_cast<float *>(d + o_ppo);
     pl->d_jobs = reinterpret_cast<Fp8StageJob *>(d + o_jobs);
     pl->d_tbt = reinterpret_cast<int32_t *>(d + o_tbt);
+    pl->d_ftok = reinterpret_cast<int32_t *>(d + o_ftok);
+    pl->d_dtok = reinterpret_cast<int32_t *>(d + o_dtok);
     pl->d_tk = d + o_tk;
     pl->d_tv = d + o_tv;
     pl->d_tq = d + o_tq;
@@ -1264,6 +1285,36 @@ int run_colocated(const fnpu_plan *pl, const AttnParams &p, void *stream) {
     return rc;
 }
 
+// A whole step whose tcgen05 prefill grid appends the prefill-path rows
+// itself (p.fa_*): the decode rows go in by a small kernel ahead of the
+// decode kernel, on the decode's stream. Co-located: the prefill grid on the
+// caller's stream, the decode stream after the fork and the prefill grid's
+// launch, as in run_colocated. Otherwise the phases one after the other.
+int run_step_fused(const fnpu_plan *pl, const AttnParams &p, const void *k_new, const void *v_new,
+                   const int64_t *slots, void *k_cache, void *v_cache, void *stream) {
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (pl->coloc) {
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_fork, s));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_fork, 0));
+        int rc = launch_prefill(pl, p, s, pl->pre_ctas, pl->e_started, false);
+        if (rc == FNPU_OK) {
+            FNPU_CUDA_TRY(cudaStreamWaitEvent(pl->s_dec, pl->e_started, 0));
+            rc = launch_kv_append_list(&pl->desc, k_new, v_new, slots, pl->d_dtok, pl->num_dtok, k_cache, v_cache,
+                                       pl->s_dec);
+        }
+        if (rc == FNPU_OK) rc = launch_decode(pl, p, pl->s_dec, 3 * pl->num_sms);
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_pre, s));
+        FNPU_CUDA_TRY(cudaEventRecord(pl->e_dec, pl->s_dec));
+        FNPU_CUDA_TRY(cudaStreamWaitEvent(s, pl->e_dec, 0));
+        return rc;
+    }
+    int rc = launch_kv_append_list(&pl->desc, k_new, v_new, slots, pl->d_dtok, pl->num_dtok, k_cache, v_cache, s);
+    if (rc == FNPU_OK && pl->num_ditems > 0)
+        rc = pl->use_dt ? launch_decode_tma(p, stream, 3 * pl->num_sms) : launch_decode_mma(p, stream);
+    if (rc != FNPU_OK) return rc;
+    return launch_prefill(pl, p, stream, pl->num_sms, nullptr, false);
+}
+
 }  // namespace
 }  // namespace fnpu
 
@@ -1283,6 +1334,46 @@ int fnpu_mixed_attn_run(const fnpu_plan *pl, const void *q, const void *k_cache,
     if (rc != FNPU_OK) return rc;
     if (pl->use_tc) return launch_prefill(pl, p, stream, pl->num_sms, nullptr, true);
     return pl->desc.kv_fp8 ? launch_prefill_fp8(p, stream) : launch_prefill_mma(p, stream);
+}
+
+int fnpu_mixed_step(const fnpu_plan *pl, const void *k_new, const void *v_new, const int64_t *slot_mapping,
+                    const void *q, void *k_cache, void *v_cache, void *out, float *lse, void *stream) {
+    if (!pl) return FNPU_EINVAL;
+    if (pl->num_tokens == 0) return FNPU_OK;
+    const bool latent = pl->desc.v_in_k_latent != 0;
+    if (!k_new || !slot_mapping || (!latent && !v_new)) return FNPU_EINVAL;
+    if (((reinterpret_cast<uintptr_t>(k_new) | (latent ? 0 : reinterpret_cast<uintptr_t>(v_new))) & 15u) ||
+        (reinterpret_cast<uintptr_t>(slot_mapping) & 7u))
+        return FNPU_EINVAL;
+    if (!run_pointers_ok(pl, q, k_cache, v_cache, out, lse)) return FNPU_EINVAL;
+    const int32_t n = static_cast<int32_t>(pl->num_tokens);
+    // the prefill grid takes the prefill rows where the plan asks for it and
+    // the prefill is the tcgen05 kernel over a bf16 cache (green-context
+    // plans keep the two calls)
+    const bool fused = (pl->flags & FNPU_PLAN_FUSED_APPEND) && pl->use_tc && !pl->use_mla && !pl->desc.kv_fp8 &&
+                       pl->num_ftok > 0 && !pl->g_pre;
+    if (!fused) {
+        const int rc = fnpu_kv_append(&pl->desc, k_new, v_new, slot_mapping, n, k_cache, v_cache, stream);
+        if (rc != FNPU_OK) return rc;
+        return fnpu_mixed_attn_run(pl, q, k_cache, v_cache, out, lse, stream);
+    }
+    AttnParams p = run_params(pl, q, k_cache, v_cache, out, lse);
+    int *range_err = nullptr;
+    const int rc = global_error_address(&range_err);
+    if (rc != FNPU_OK) return rc;
+    p.fa_k_new = static_cast<const uint4 *>(k_new);
+    p.fa_v_new = static_cast<const uint4 *>(v_new);
+    p.fa_slots = slot_mapping;
+    p.fa_tokens = pl->d_ftok;
+    p.fa_k_cache = static_cast<uint4 *>(k_cache);
+    p.fa_v_cache = static_cast<uint4 *>(v_cache);
+    p.fa_count = pl->d_err + 6;  // zero between runs (the last CTA out resets it)
+    p.fa_range_err = range_err;
+    p.fa_num_tokens = pl->num_ftok;
+    p.fa_k_chunks = static_cast<int32_t>(static_cast<int64_t>(pl->desc.num_kv_heads) * pl->desc.head_dim_qk * 2 / 16);
+    p.fa_v_chunks = static_cast<int32_t>(static_cast<int64_t>(pl->desc.num_kv_heads) * pl->desc.head_dim_v * 2 / 16);
+    p.fa_num_slots = static_cast<int64_t>(pl->desc.num_blocks) * pl->desc.block_size;
+    return run_step_fused(pl, p, k_new, v_new, slot_mapping, k_cache, v_cache, stream);
 }
 
 int fnpu_plan_check(const fnpu_plan *pl, void *stream) {

@@ -102,6 +102,20 @@ struct AttnParams {
     int32_t num_mitems;
     int32_t *err;           // device error flag of the plan
     int32_t *sched;         // persistent work queues: [0..1] prefill, [2..3] decode (next item, finished CTAs)
+    // the step's append of the prefill-path rows inside the tcgen05 prefill
+    // (fnpu_mixed_step): fa_count null = none. Tokens fa_tokens[0 .. n) of
+    // k_new / v_new go to their slots; a grid-wide count (zero between runs)
+    // says when every CTA has written its share.
+    const uint4 *fa_k_new;
+    const uint4 *fa_v_new;
+    const int64_t *fa_slots;
+    const int32_t *fa_tokens;
+    uint4 *fa_k_cache;
+    uint4 *fa_v_cache;
+    int32_t *fa_count;
+    int *fa_range_err;      // the library-wide error flag (bit 0: a slot past the pool)
+    int32_t fa_num_tokens, fa_k_chunks, fa_v_chunks;
+    int64_t fa_num_slots;
 };
 
 // cuTensorMapEncodeTiled, looked up once through the runtime's driver entry
@@ -124,6 +138,9 @@ int cuda_fail(cudaError_t e, const char *where);
 int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_new,
                      const int64_t *slots, int32_t num_tokens, void *k_cache, void *v_cache,
                      void *stream);
+// the same append for the tokens tokens[0 .. n) of k_new / v_new only
+int launch_kv_append_list(const fnpu_attn_desc *d, const void *k_new, const void *v_new, const int64_t *slots,
+                          const int32_t *tokens, int32_t n, void *k_cache, void *v_cache, void *stream);
 int read_and_clear_global_error(void *stream, int *flag);
 // Device address of the library-wide error flag on the current device (looked
 // up once per device), for kernels of other translation units that raise it.
@@ -162,7 +179,9 @@ bool mla_supported(int d_qk, int d_v, int hq, int hkv);
 int mla_heads_per_item();
 // started (a cudaEvent_t, may be null): recorded once every CTA has begun;
 // f16: Q, K and V are f16 (d = 128 only), else bf16; pdl: a programmatic
-// dependent launch of the kernel before it on `stream`
+// dependent launch of the kernel before it on `stream`. With p.fa_count set
+// the CTAs first write the prefill-path rows of the step (a cooperative
+// launch: they wait for one another before reading the cache).
 int launch_prefill_tc(const AttnParams &p, void *stream, int max_ctas, void *started = nullptr, bool f16 = false,
                       bool pdl = false);
 bool prefill_tc_supported(int d_qk, int d_v, int block_size, int group);

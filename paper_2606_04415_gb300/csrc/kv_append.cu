@@ -164,6 +164,46 @@ int launch_kv_append(const fnpu_attn_desc *d, const void *k_new, const void *v_n
     return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
 }
 
+// The append of listed tokens only (the decode rows of a step whose prefill
+// grid appends the prefill rows itself): chunk i belongs to token
+// tokens[i / (k_chunks + v_chunks)].
+__global__ void __launch_bounds__(256) kv_append_list_kernel(
+    const uint4 *__restrict__ k_new, const uint4 *__restrict__ v_new, const int64_t *__restrict__ slots,
+    const int32_t *__restrict__ tokens, int32_t n, int32_t k_chunks, int32_t v_chunks, uint4 *__restrict__ k_cache,
+    uint4 *__restrict__ v_cache, int64_t num_slots) {
+    const int32_t per_tok = k_chunks + v_chunks;
+    const int64_t total = static_cast<int64_t>(n) * per_tok;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int32_t ti = static_cast<int32_t>(i / per_tok);
+        const int32_t c = static_cast<int32_t>(i - static_cast<int64_t>(ti) * per_tok);
+        const int64_t t = __ldg(tokens + ti);
+        const uint4 v = c < k_chunks ? __ldg(k_new + t * k_chunks + c) : __ldg(v_new + t * v_chunks + (c - k_chunks));
+        const int64_t s = __ldg(slots + t);
+        if (s < 0) continue;
+        if (s >= num_slots) {
+            if (c == 0) atomicOr(&g_device_error, 1);
+            continue;
+        }
+        if (c < k_chunks) k_cache[s * k_chunks + c] = v;
+        else v_cache[s * v_chunks + (c - k_chunks)] = v;
+    }
+}
+
+int launch_kv_append_list(const fnpu_attn_desc *d, const void *k_new, const void *v_new, const int64_t *slots,
+                          const int32_t *tokens, int32_t n, void *k_cache, void *v_cache, void *stream) {
+    if (n == 0) return FNPU_OK;
+    const int32_t kc = static_cast<int32_t>(static_cast<int64_t>(d->num_kv_heads) * d->head_dim_qk * 2 / 16);
+    const int32_t vc = static_cast<int32_t>(static_cast<int64_t>(d->num_kv_heads) * d->head_dim_v * 2 / 16);
+    const int64_t want = (static_cast<int64_t>(n) * (kc + vc) + 255) / 256;
+    const int grid = static_cast<int>(want < 4096 ? want : 4096);
+    kv_append_list_kernel<<<grid, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint4 *>(k_new), static_cast<const uint4 *>(v_new), slots, tokens, n, kc, vc,
+        static_cast<uint4 *>(k_cache), static_cast<uint4 *>(v_cache),
+        static_cast<int64_t>(d->num_blocks) * d->block_size);
+    return cudaGetLastError() == cudaSuccess ? FNPU_OK : FNPU_ECUDA;
+}
+
 // One warp per row: the 64 16-byte chunks of c into the workspace (two per
 // lane), then the 8 chunks of r into every head's key (lane e writes chunk
 // e mod 8 of heads e / 8, e / 8 + 4, ...). A negative slot gives a zero row;

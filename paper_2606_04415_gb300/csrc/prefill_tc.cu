@@ -123,6 +123,54 @@ __device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, int idx) {
     return g;
 }
 
+// The step's append of the prefill-path rows inside the prefill grid
+// (fnpu_mixed_step; both phases share the KV pool, Sec. 3.4), shared by the
+// CTAs: 16-byte chunks, consecutive threads on consecutive chunks of a row,
+// the row and its slot loaded together. Then every CTA waits (bounded) until
+// all have written theirs, before any warp reads the cache; the launch is
+// cooperative, so all are resident. False if the wait ran out (the plan's
+// error flag is raised). A call of its own, so that the kernel's warps keep
+// their register allocation.
+__device__ __noinline__ bool fused_append(const AttnParams &p, int tid) {
+    const int32_t kc = p.fa_k_chunks, per_tok = kc + p.fa_v_chunks;
+    const int64_t total = static_cast<int64_t>(p.fa_num_tokens) * per_tok;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + tid; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int32_t ti = static_cast<int32_t>(i / per_tok);
+        const int32_t c = static_cast<int32_t>(i - static_cast<int64_t>(ti) * per_tok);
+        const int64_t t = __ldg(p.fa_tokens + ti);
+        const uint4 v = c < kc ? __ldg(p.fa_k_new + t * kc + c) : __ldg(p.fa_v_new + t * p.fa_v_chunks + (c - kc));
+        const int64_t s = __ldg(p.fa_slots + t);
+        if (s < 0) continue;  // padding
+        if (s >= p.fa_num_slots) {
+            if (c == 0) atomicOr(p.fa_range_err, 1);
+            continue;
+        }
+        if (c < kc) p.fa_k_cache[s * kc + c] = v;
+        else p.fa_v_cache[s * p.fa_v_chunks + (c - kc)] = v;
+    }
+    tc::fence_proxy_async_global();  // before the TMA reads of the rows, here and in other CTAs
+    __syncthreads();
+    __shared__ int ok_all;
+    if (tid == 0) {
+        __threadfence();
+        atomicAdd(p.fa_count, 1);
+        int spins = 0, ok = 1;
+        while (tc::ld_acquire_gpu(p.fa_count) < static_cast<int>(gridDim.x)) {
+            if (++spins > (1 << 22)) {  // a CTA that never came: flag it, and leave the work undone
+                atomicOr(p.err, 1);
+                ok = 0;
+                break;
+            }
+            __nanosleep(32);
+        }
+        tc::fence_proxy_async_global();
+        ok_all = ok;
+    }
+    __syncthreads();
+    return ok_all != 0;
+}
+
 // F16: the operands (Q, K, V and P) are f16 instead of bf16 (the FP8 cache's
 // prefill: its codes are dequantised to f16 first)
 template <int DQ, int DV, bool F16>
@@ -190,6 +238,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = *tmem_slot;
+
+    if (p.fa_count != nullptr && !fused_append(p, tid)) *abort_flag = 1;
 
     auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
         if (tc::mbar_try_wait(bar, parity)) return true;
@@ -650,11 +700,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, kTmemCols);
     }
-    if (tid == 0) {  // the last CTA out resets the work queue for the next run
+    if (tid == 0) {  // the last CTA out resets the work queue (and the append count) for the next run
         __threadfence();
         if (atomicAdd(p.sched + 1, 1) == static_cast<int>(gridDim.x) - 1) {
             p.sched[0] = 0;
             p.sched[1] = 0;
+            if (p.fa_count != nullptr) *p.fa_count = 0;
             __threadfence();
         }
     }
@@ -705,7 +756,8 @@ int launch_tc(const AttnParams &p, cudaStream_t st, int max_ctas, cudaEvent_t st
     FNPU_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                                        cudaSharedmemCarveoutMaxShared));
     const int grid = p.num_pitems < max_ctas ? p.num_pitems : max_ctas;
-    FNPU_CUDA_TRY(launch_ex(kernel, grid, kThreads, Cfg::kSmemBytes, st, pdl, started, p, maps));
+    FNPU_CUDA_TRY(launch_coop(kernel, grid, kThreads, Cfg::kSmemBytes, st, pdl, started, p.fa_count != nullptr, p,
+                              maps));
     return FNPU_OK;
 }
 

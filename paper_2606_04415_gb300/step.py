@@ -18,7 +18,7 @@ from typing import Optional
 import numpy as np
 
 from . import (FP8_BLOCK_BYTES, PlanOpts, kv_append, make_desc, mixed_attn_plan, mixed_attn_replan,
-               mixed_attn_run)
+               mixed_attn_run, mixed_step)
 
 
 def _to_dev(a: Optional[np.ndarray], torch, dtype, device):
@@ -96,9 +96,11 @@ class DeviceStep:
                        stream=stream)
 
     def run(self, stream=None):
-        """One step: append the new tokens, then attention."""
-        self.append(stream)
-        self.attend(stream)
+        """One step: the append of the new tokens and the attention, in one
+        call (``fnpu_mixed_step``; the same results as ``append`` then
+        ``attend``)."""
+        mixed_step(self.plan, self.k_new, self.v_new, self.slot_mapping, self.q, self.k_cache, self.v_cache,
+                   self.out, self.lse, stream=stream)
 
     def results(self):
         """(out float32 numpy, lse float32 numpy) after synchronising."""
