@@ -51,7 +51,7 @@ L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 # workload whose kernels change until they are captured again.
 NCU_TRAFFIC = {
     # co-located workloads: the prefill kernel (the dominant one), captured alone
-    "qwen_coloc": 33.5e6,        # prefill_tc 33.3 MB read + 0.21 MB write
+    "qwen_coloc": 33.6e6,        # prefill_tc 33.3 MB read + 0.32 MB write
     "qwen_decode": 308.9e6,      # decode_tma 308.15 MB read + 0.7 MB write
     "qwen_decode_fp8": 159.6e6,  # decode_fp8 159.16 MB read + 0.4 MB write
     "mla_prefill_expand": 203.4e6,  # prefill_tc<192, 128> 188.9 MB read + 14.5 MB write
