@@ -54,7 +54,7 @@ NCU_TRAFFIC = {
     "qwen_coloc": 33.6e6,        # prefill_tc 33.3 MB read + 0.32 MB write
     "qwen_decode": 308.9e6,      # decode_tma 308.15 MB read + 0.7 MB write
     "qwen_decode_fp8": 159.6e6,  # decode_fp8 159.16 MB read + 0.4 MB write
-    "mla_prefill_expand": 203.4e6,  # prefill_tc<192, 128> 188.9 MB read + 14.5 MB write
+    "mla_prefill_expand": 200.9e6,  # prefill_tc<192, 128> 186.8 MB read + 14.0 MB write
 }
 
 
