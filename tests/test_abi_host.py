@@ -124,6 +124,7 @@ def test_append_and_run_reject_null_pointers():
     assert lib.fnpu_mixed_attn_replan(None, 0, None, None, None, None, 1, None, None) == fnpu.FNPU_EINVAL
     share = ctypes.c_int32(-1)
     assert lib.fnpu_plan_decode_share(None, ctypes.byref(share)) == fnpu.FNPU_EINVAL and share.value == -1
+    assert lib.fnpu_mixed_step(None, 16, 32, 64, 128, 256, 512, 1024, 2048, None) == fnpu.FNPU_EINVAL
     lib.fnpu_plan_destroy(None)  # ignored
 
 
