@@ -44,7 +44,9 @@
 // Launched as a programmatic dependent of the kernel before it (the step's
 // KV append), the grid sets up while that kernel drains; the two loader
 // warps wait for it (griddepcontrol.wait) before their first read, and every
-// other warp reads global memory only after them.
+// other warp reads global memory only after them. Optionally (a cooperative
+// launch, fused_append) the CTAs write the step's prefill rows into the cache
+// themselves first and wait for one another before any warp takes its role.
 #include <math.h>
 
 #include "common.cuh"
