@@ -181,3 +181,16 @@ def test_out_of_range_slot_gives_zero_row_and_flag():
     fnpu.mla_expand(st.latent_desc, st.latent, bad, st.w_uk, st.w_uv, ws, k, v)
     assert fnpu.check() == fnpu.FNPU_EDEVICE_RANGE
     assert not k.float().abs().sum().item() and not v.float().abs().sum().item()
+
+
+@pytest.mark.parametrize("case", range(4))
+def test_random_chunks_on_prefixes(case):
+    """Random chunk lengths (1 to 160 rows), prefixes (0 to 500), latent block
+    sizes and head counts, on the tcgen05 and the mma.sync attention; every
+    row within the derived bounds."""
+    rng = np.random.default_rng(900 + case)
+    S = int(rng.integers(1, 4))
+    q = [int(rng.integers(1, 161)) for _ in range(S)]
+    ctx = [x + int(rng.integers(0, 501)) for x in q]
+    _run(q, ctx, heads=int(rng.choice([16, 128])), seed=20 + case, bs=int(rng.choice([16, 32, 64])),
+         flags=int(rng.choice([0, 2])))
